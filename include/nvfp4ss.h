@@ -1,0 +1,154 @@
+/*
+ * nvfp4ss.h -- C ABI of libnvfp4ss.so: NVFP4 quantisation with ScaleSweep block
+ * scales on NVIDIA GB300 (sm_103a).
+ *
+ * Method: "ScaleSweep: Accurate NVFP4 Post-Training Quantization of LLMs via
+ * Block Scale Initialization".  A tensor x is represented as (q, s, S): FP4 E2M1
+ * elements q, one FP8 E4M3 scale s per block of consecutive elements and one
+ * FP32 global scale S, with x_hat_i = q_i * s_{i/block} * S (Sec. 3.2).
+ *
+ * Conventions shared by every entry point
+ *   - Tensors are row-major [rows, cols]; blocks run along cols (the input
+ *     channel of a [out, in] linear weight), so cols % block == 0.
+ *   - All tensor pointers are device-accessible pointers (cudaMalloc, torch
+ *     CUDA tensors, managed or registered host memory).  The caller allocates
+ *     and owns every buffer; the library never allocates, frees or synchronises.
+ *   - Every call is asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *     default stream).  S is read from device memory by the kernels, so a
+ *     per-call global scale needs no host round trip.
+ *   - Argument, shape and alignment errors are detected on the host before any
+ *     launch and returned as a status; nothing is launched then.  A failed
+ *     launch returns NVFP4_ERR_CUDA.  Data errors (NaN/inf input) are reported
+ *     through the device status word of nvfp4_global_scale.
+ *   - Packed FP4 layout: codes[rows, cols/2] bytes, element 2j in the low
+ *     nibble and element 2j+1 in the high nibble; a nibble is sign (bit 3) and
+ *     the 3-bit E2M1 magnitude code (0, 0.5, 1, 1.5, 2, 3, 4, 6).
+ *   - Scale layouts: linear sf[rows, cols/block] E4M3 codes; swizzled (block 16
+ *     only) is the 128x4-atom layout read by tcgen05 block-scaled MMA:
+ *     ceil(rows/128)*128 x ceil(cols/64)*4 bytes, atom (row/128, col4/4) at
+ *     ((row/128)*ceil(kb/4) + k/4)*512, inside it (row%32)*16 + ((row/32)%4)*4 + k%4;
+ *     padding bytes are written as 0.
+ *
+ * Arithmetic contract (where the paper fixes no arithmetic; decisions in fp32):
+ *   E = fl(1/S), y = fl(x*E); m = max|y| per block; s_base = fl(m/6);
+ *   I0 = code of floor_E4M3(s_base); candidate c: t = fl(y*fl(1/v_c)),
+ *   q = RNE_E2M1(t) saturating at 6; loss L_c = sum w (y - q v_c)^2;
+ *   argmin over the window with exact ties going to the lowest code.
+ *   A block with m == 0, or any block when S is not a positive finite float
+ *   with finite 1/S, gets scale code 0 and nibbles carrying only the sign of x.
+ */
+#ifndef NVFP4SS_H
+#define NVFP4SS_H
+
+#include <limits.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    NVFP4_OK = 0,
+    NVFP4_ERR_INVALID_ARG = 1,   /* null/overlapping pointer, bad enum, bad shape or window */
+    NVFP4_ERR_UNSUPPORTED = 2,   /* block not in {16,32,64}; swizzled scales with block != 16 */
+    NVFP4_ERR_ALIGNMENT = 3,     /* a pointer misses its required alignment */
+    NVFP4_ERR_RANGE = 4,         /* a size overflows int64 or the device limits */
+    NVFP4_ERR_CUDA = 5           /* a CUDA runtime call or launch failed */
+} nvfp4_status;
+
+typedef enum { NVFP4_IN_BF16 = 0, NVFP4_IN_F32 = 1 } nvfp4_dtype;
+typedef enum { NVFP4_OBJ_MSE = 0, NVFP4_OBJ_WMSE = 1 } nvfp4_objective;
+typedef enum { NVFP4_SF_LINEAR = 1, NVFP4_SF_SWIZZLED = 2 } nvfp4_sf_layout;
+
+/* Pass as win_lo and win_hi to use the paper's window (Sec. 4.2.2). */
+#define NVFP4_WINDOW_DEFAULT INT_MIN
+
+/* Human-readable name of a status code (static storage). */
+const char* nvfp4_status_string(nvfp4_status st);
+
+/*
+ * Bytes of device workspace nvfp4_global_scale needs for n elements.
+ */
+size_t nvfp4_global_scale_workspace(int64_t n);
+
+/*
+ * Global scale S = fl32(amax / fl32(6*fp8_div)), amax = max_i |x_i| (Sec. 3.2
+ * with fp8_div = 448, AbsMax; Sec. 4.2.1 with fp8_div = 256, ScaleSweep).
+ *   x          [n] elements of type dt, 16-byte aligned.
+ *   S_out      device float written with S.
+ *   status_dev optional device int; bit 0 is OR-ed in if x holds NaN or inf
+ *              (NaNs are ignored by the max, an inf makes S = inf).
+ *   workspace  device scratch of nvfp4_global_scale_workspace(n) bytes,
+ *              16-byte aligned; its contents need no initialisation.
+ * n == 0 writes S = 0.  Two kernel launches on `stream`.
+ */
+nvfp4_status nvfp4_global_scale(const void* x, nvfp4_dtype dt, int64_t n, float fp8_div, float* S_out,
+                                int* status_dev, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * ScaleSweep quantisation (Sec. 4.2.2): per block, sweep the E4M3 scale codes
+ * in [I0 + win_lo, I0 + win_hi] (clamped to 1..126), score each with the MSE
+ * (Sec. 4.1, Eq. for L^MSE) or WMSE (Sec. 4.1, diagonal-Gram importance)
+ * objective, keep the argmin (exact ties -> lowest code) and emit its codes.
+ *   x             [rows, cols] of type dt, 16-byte aligned.
+ *   block         16, 32 or 64 elements per scale.
+ *   S             device float (global scale, e.g. from nvfp4_global_scale).
+ *   obj, w        NVFP4_OBJ_WMSE reads per-element weights w[row*w_row_stride + col]
+ *                 (float, >= 0, 16-byte aligned; w_row_stride = 0 broadcasts one
+ *                 [cols] vector, e.g. per-input-channel importance ||X[:,i]||^2);
+ *                 w is ignored for MSE and may be NULL.
+ *   win_lo/hi     bit-pattern offsets, -126 <= win_lo <= win_hi <= 126, or both
+ *                 NVFP4_WINDOW_DEFAULT: [-3, 7] for MSE with block 16 (Lemma 4.3),
+ *                 [-8, 7] otherwise (WMSE: empirical s_base/2; blocks of 32/64:
+ *                 the paper gives no window).  (-126, 126) is the exhaustive sweep.
+ *   codes         [rows, cols/2] packed nibbles, 8-byte aligned.
+ *   sf_linear     optional [rows, cols/block] scale codes.
+ *   sf_swizzled   optional 128x4-atom scale layout (block 16 only).
+ *                 At least one of sf_linear / sf_swizzled must be given.
+ *   block_loss    optional [rows*cols/block] float: the chosen candidate's loss in
+ *                 the S-normalised domain (multiply by S^2 for the x domain).
+ * Outputs must not overlap x, w or each other.
+ */
+nvfp4_status scalesweep_quantize(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                                 const float* S, nvfp4_objective obj, const float* w, int64_t w_row_stride,
+                                 int win_lo, int win_hi, uint8_t* codes, uint8_t* sf_linear,
+                                 uint8_t* sf_swizzled, float* block_loss, void* stream);
+
+/*
+ * AbsMax quantisation (Sec. 3.2): s = max(1, RN_E4M3(s_base)) as a code (a block
+ * whose RN scale would be 0 gets the smallest positive scale), q = RNE_E2M1.
+ * Arguments as scalesweep_quantize; block_loss is the MSE loss of the chosen
+ * scale.  This is the baseline the overhead of the sweep is measured against.
+ */
+nvfp4_status absmax_quantize(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                             const float* S, uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled,
+                             float* block_loss, void* stream);
+
+/*
+ * 4/6 quantisation (Sec. 2, FP4 quantization): besides the AbsMax scale c6, try
+ * c4 = max(1, RN_E4M3(fl(m/4))) (block max mapped to 4) and keep c4 only if its
+ * loss under `obj` is strictly lower.  Arguments as scalesweep_quantize.
+ */
+nvfp4_status four_over_six_quantize(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                                    const float* S, nvfp4_objective obj, const float* w, int64_t w_row_stride,
+                                    uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled,
+                                    float* block_loss, void* stream);
+
+/*
+ * Dequantisation x_hat = fl32(fl32(q * s) * S) (Sec. 3.2 reconstruction; the
+ * simulated quantisation of Sec. 5.1), written as fp32 or as the RNE bf16 of
+ * that fp32 value.
+ *   codes  [rows, cols/2] packed nibbles (8-byte aligned); sf in `layout`
+ *   (NVFP4_SF_SWIZZLED requires block 16); out [rows, cols] of out_dt,
+ *   16-byte aligned.
+ */
+nvfp4_status nvfp4_dequantize(const uint8_t* codes, const uint8_t* sf, nvfp4_sf_layout layout, const float* S,
+                              int64_t rows, int64_t cols, int block, void* out, nvfp4_dtype out_dt,
+                              void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* NVFP4SS_H */

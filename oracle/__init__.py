@@ -59,7 +59,7 @@ def _load(path: str) -> ctypes.CDLL:
     L.oracle_global_scale.argtypes = [c_p, c_i64, c_f, c_p, c_p]
     L.oracle_quantize.argtypes = [c_i, c_p, c_i64, c_i64, c_i, c_f, c_i, c_p, c_i64, c_i, c_i,
                                   c_p, c_p, c_p, c_p, c_p, c_i, c_p, c_i]
-    L.oracle_block_losses_at.argtypes = [c_p, c_i64, c_i64, c_i, c_f, c_i, c_p, c_i64, c_p, c_p, c_i]
+    L.oracle_block_losses_at.argtypes = [c_p, c_i64, c_i64, c_i, c_f, c_i, c_p, c_i64, c_p, c_p, c_p, c_i]
     L.oracle_swizzle_offset.argtypes, L.oracle_swizzle_offset.restype = [c_i64, c_i64, c_i64], c_i64
     L.oracle_swizzle_bytes.argtypes, L.oracle_swizzle_bytes.restype = [c_i64, c_i64], c_i64
     L.oracle_swizzle_scales.argtypes = [c_p, c_i64, c_i64, c_p]
@@ -180,19 +180,22 @@ def quantize(method: int, x: np.ndarray, block: int, S: float, objective: int = 
 
 
 def block_losses_at(x: np.ndarray, block: int, S: float, sf_codes: np.ndarray, objective: int = MSE,
-                    w: np.ndarray | None = None, w_row_stride: int = 0, nthreads: int = 0) -> np.ndarray:
-    """float64 loss of each block under the given scale codes (same contract)."""
+                    w: np.ndarray | None = None, w_row_stride: int = 0, nthreads: int = 0,
+                    want_codes: bool = False):
+    """float64 loss of each block under the given scale codes (same contract);
+    with want_codes also the packed nibbles those scales produce."""
     x = np.ascontiguousarray(x, dtype=np.float32)
     rows, cols = x.shape
     sfc = np.ascontiguousarray(sf_codes, dtype=np.uint8).reshape(-1)
     out = np.zeros(rows * (cols // block), np.float64)
+    codes = np.zeros((rows, cols // 2), np.uint8) if want_codes else None
     if w is not None:
         w = np.ascontiguousarray(w, dtype=np.float32)
     rc = lib().oracle_block_losses_at(_ptr(x), rows, cols, block, float(np.float32(S)), objective, _ptr(w),
-                                      int(w_row_stride), _ptr(sfc), _ptr(out), int(nthreads))
+                                      int(w_row_stride), _ptr(sfc), _ptr(out), _ptr(codes), int(nthreads))
     if rc != 0:
         raise ValueError("oracle_block_losses_at: bad arguments")
-    return out
+    return (out, codes) if want_codes else out
 
 
 def swizzle_bytes(rows: int, kblocks: int) -> int:

@@ -284,10 +284,11 @@ int oracle_quantize(int method, const float* x, int64_t rows, int64_t cols, int 
     return 0;
 }
 
-/* Loss of a given code on every block (used to score a GPU pick). */
+/* Loss of a given scale code on every block, and optionally the packed
+ * nibbles it yields (used to score and check a GPU pick on a near-tie). */
 int oracle_block_losses_at(const float* x, int64_t rows, int64_t cols, int block, float S,
                            int objective, const float* w, int64_t w_row_stride,
-                           const uint8_t* sf_codes, double* out, int nthreads)
+                           const uint8_t* sf_codes, double* out, uint8_t* codes_out, int nthreads)
 {
     if (block <= 0 || block > 64 || cols % block != 0) return -1;
     int64_t kb = cols / block, nblocks = rows * kb;
@@ -302,14 +303,23 @@ int oracle_block_losses_at(const float* x, int64_t rows, int64_t cols, int block
         const float* xb = x + row * cols + kbi * block;
         const float* wb = (objective == ORACLE_WMSE) ? (w + row * w_row_stride + kbi * block) : NULL;
         float y[64];
+        uint8_t q[64];
         for (int i = 0; i < block; i++) y[i] = usable ? xb[i] * E : xb[i];
         int c = sf_codes[blk] & 0x7F;
         if (c == 0 || c == 127) {
             double L = 0.0;
-            for (int i = 0; i < block; i++) L += (wb ? (double)wb[i] : 1.0) * (double)y[i] * (double)y[i];
+            for (int i = 0; i < block; i++) {
+                L += (wb ? (double)wb[i] : 1.0) * (double)y[i] * (double)y[i];
+                q[i] = signbit(y[i]) ? 8 : 0;
+            }
             out[blk] = L;
         } else {
-            out[blk] = block_loss(y, wb, block, c, NULL);
+            out[blk] = block_loss(y, wb, block, c, q);
+        }
+        if (codes_out) {
+            uint8_t* cb = codes_out + row * (cols / 2) + kbi * (block / 2);
+            for (int j = 0; j < block / 2; j++)
+                cb[j] = (uint8_t)((q[2 * j] & 0xF) | ((q[2 * j + 1] & 0xF) << 4));
         }
     }
     return 0;

@@ -1,0 +1,153 @@
+"""Thin ctypes binding of libnvfp4ss.so (include/nvfp4ss.h).
+
+Every function has the name of the C entry point it calls and only marshals
+arguments: torch CUDA tensors become device pointers, the current torch CUDA
+stream becomes the cudaStream_t, a non-OK status raises ``Nvfp4Error``.  All
+arithmetic runs in the library's CUDA kernels; there is no CPU fallback, and a
+missing library raises at load time.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import build as _build
+
+NVFP4_IN_BF16, NVFP4_IN_F32 = 0, 1
+NVFP4_OBJ_MSE, NVFP4_OBJ_WMSE = 0, 1
+NVFP4_SF_LINEAR, NVFP4_SF_SWIZZLED = 1, 2
+NVFP4_WINDOW_DEFAULT = -(2 ** 31)
+
+STATUS = {0: "NVFP4_OK", 1: "NVFP4_ERR_INVALID_ARG", 2: "NVFP4_ERR_UNSUPPORTED", 3: "NVFP4_ERR_ALIGNMENT",
+          4: "NVFP4_ERR_RANGE", 5: "NVFP4_ERR_CUDA"}
+
+
+class Nvfp4Error(RuntimeError):
+    def __init__(self, fn: str, code: int, msg: str):
+        super().__init__(f"{fn}: {STATUS.get(code, code)} ({msg})")
+        self.code = code
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def lib() -> ctypes.CDLL:
+    """Load libnvfp4ss.so, building it first if it is missing or stale."""
+    global _lib
+    if _lib is None:
+        if not _build.up_to_date():
+            _build.build()
+        if not os.path.exists(_build.LIB):
+            raise RuntimeError("libnvfp4ss.so is not built and could not be built")
+        L = ctypes.CDLL(_build.LIB)
+        i, i64, f, p, sz = ctypes.c_int, ctypes.c_int64, ctypes.c_float, ctypes.c_void_p, ctypes.c_size_t
+        L.nvfp4_status_string.argtypes, L.nvfp4_status_string.restype = [i], ctypes.c_char_p
+        L.nvfp4_global_scale_workspace.argtypes, L.nvfp4_global_scale_workspace.restype = [i64], sz
+        L.nvfp4_global_scale.argtypes = [p, i, i64, f, p, p, p, sz, p]
+        L.scalesweep_quantize.argtypes = [p, i, i64, i64, i, p, i, p, i64, i, i, p, p, p, p, p]
+        L.absmax_quantize.argtypes = [p, i, i64, i64, i, p, p, p, p, p, p]
+        L.four_over_six_quantize.argtypes = [p, i, i64, i64, i, p, i, p, i64, p, p, p, p, p]
+        L.nvfp4_dequantize.argtypes = [p, p, i, p, i64, i64, i, p, i, p]
+        for fn in ("nvfp4_global_scale", "scalesweep_quantize", "absmax_quantize", "four_over_six_quantize",
+                   "nvfp4_dequantize"):
+            getattr(L, fn).restype = i
+        _lib = L
+    return _lib
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return ctypes.c_void_p(t)
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, torch.cuda.Stream):
+        return ctypes.c_void_p(stream.cuda_stream)
+    return ctypes.c_void_p(int(stream))
+
+
+def _dtype(x) -> int:
+    if x.dtype == torch.bfloat16:
+        return NVFP4_IN_BF16
+    if x.dtype == torch.float32:
+        return NVFP4_IN_F32
+    raise TypeError(f"unsupported dtype {x.dtype}")
+
+
+def _check(fn: str, rc: int):
+    if rc != 0:
+        raise Nvfp4Error(fn, rc, lib().nvfp4_status_string(rc).decode())
+
+
+def nvfp4_status_string(code: int) -> str:
+    return lib().nvfp4_status_string(int(code)).decode()
+
+
+def nvfp4_global_scale_workspace(n: int) -> int:
+    return int(lib().nvfp4_global_scale_workspace(int(n)))
+
+
+def nvfp4_global_scale(x, fp8_div: float, S_out, status=None, workspace=None, stream=None):
+    ws_bytes = workspace.numel() * workspace.element_size()
+    rc = lib().nvfp4_global_scale(_ptr(x), _dtype(x), x.numel(), float(fp8_div), _ptr(S_out), _ptr(status),
+                                  _ptr(workspace), ws_bytes, _stream(stream))
+    _check("nvfp4_global_scale", rc)
+
+
+def scalesweep_quantize(x, block: int, S, objective: int, w, w_row_stride: int, win_lo: int, win_hi: int,
+                        codes, sf_linear=None, sf_swizzled=None, block_loss=None, stream=None):
+    rows, cols = x.shape
+    rc = lib().scalesweep_quantize(_ptr(x), _dtype(x), rows, cols, int(block), _ptr(S), int(objective), _ptr(w),
+                                   int(w_row_stride), int(win_lo), int(win_hi), _ptr(codes), _ptr(sf_linear),
+                                   _ptr(sf_swizzled), _ptr(block_loss), _stream(stream))
+    _check("scalesweep_quantize", rc)
+
+
+def absmax_quantize(x, block: int, S, codes, sf_linear=None, sf_swizzled=None, block_loss=None, stream=None):
+    rows, cols = x.shape
+    rc = lib().absmax_quantize(_ptr(x), _dtype(x), rows, cols, int(block), _ptr(S), _ptr(codes), _ptr(sf_linear),
+                               _ptr(sf_swizzled), _ptr(block_loss), _stream(stream))
+    _check("absmax_quantize", rc)
+
+
+def four_over_six_quantize(x, block: int, S, objective: int, w, w_row_stride: int, codes, sf_linear=None,
+                           sf_swizzled=None, block_loss=None, stream=None):
+    rows, cols = x.shape
+    rc = lib().four_over_six_quantize(_ptr(x), _dtype(x), rows, cols, int(block), _ptr(S), int(objective), _ptr(w),
+                                      int(w_row_stride), _ptr(codes), _ptr(sf_linear), _ptr(sf_swizzled),
+                                      _ptr(block_loss), _stream(stream))
+    _check("four_over_six_quantize", rc)
+
+
+def nvfp4_dequantize(codes, sf, layout: int, S, rows: int, cols: int, block: int, out, stream=None):
+    rc = lib().nvfp4_dequantize(_ptr(codes), _ptr(sf), int(layout), _ptr(S), int(rows), int(cols), int(block),
+                                _ptr(out), _dtype(out), _stream(stream))
+    _check("nvfp4_dequantize", rc)
+
+
+# --------------------------------------------------------------------------- buffer helpers
+def swizzled_bytes(rows: int, cols: int, block: int = 16) -> int:
+    kb = cols // block
+    return -(-rows // 128) * 128 * (-(-kb // 4)) * 4
+
+
+def empty_outputs(rows: int, cols: int, block: int, device="cuda", linear=True, swizzled=False, loss=False) -> dict:
+    """Allocate the output buffers of a quantise call with torch (the library
+    itself never allocates)."""
+    out = {"codes": torch.empty(rows, cols // 2, dtype=torch.uint8, device=device)}
+    out["sf_linear"] = torch.empty(rows, cols // block, dtype=torch.uint8, device=device) if linear else None
+    out["sf_swizzled"] = torch.empty(swizzled_bytes(rows, cols, block), dtype=torch.uint8, device=device) \
+        if swizzled else None
+    out["block_loss"] = torch.empty(rows * (cols // block), dtype=torch.float32, device=device) if loss else None
+    return out

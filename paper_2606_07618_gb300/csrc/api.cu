@@ -1,0 +1,264 @@
+// Host side of the C ABI declared in include/nvfp4ss.h: argument, alignment and
+// overlap checks (all before any launch), then dispatch to the kernels.  The
+// library never allocates, frees or synchronises; every call is asynchronous on
+// the caller's stream.
+#include <climits>
+#include <cstdint>
+#include <cstring>
+
+#include <cuda_runtime.h>
+
+#include "nvfp4_kernels.h"
+#include "nvfp4ss.h"
+
+using namespace nvfp4;
+
+namespace {
+
+int sm_count() {
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 0;
+    if (dev < 64 && cache[dev] > 0) return cache[dev];
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    if (dev < 64) cache[dev] = n;
+    return n;
+}
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+bool mul_ok(int64_t a, int64_t b, int64_t* out) {
+    if (a < 0 || b < 0) return false;
+    if (a != 0 && b > INT64_MAX / a) return false;
+    *out = a * b;
+    return true;
+}
+
+// [p, p+n) and [q, q+m) overlap?
+bool overlap(const void* p, int64_t n, const void* q, int64_t m) {
+    if (!p || !q || n <= 0 || m <= 0) return false;
+    uintptr_t a = reinterpret_cast<uintptr_t>(p), b = reinterpret_cast<uintptr_t>(q);
+    return a < b + (uintptr_t)m && b < a + (uintptr_t)n;
+}
+
+// The kernels dereference these pointers on the device: reject memory the GPU
+// cannot address (plain pageable host memory or garbage) before launching.
+bool device_accessible(const void* p) {
+    if (!p) return true;
+    cudaPointerAttributes at;
+    cudaError_t e = cudaPointerGetAttributes(&at, p);
+    if (e != cudaSuccess) {
+        (void)cudaGetLastError();
+        return false;
+    }
+    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged ||
+           (at.type == cudaMemoryTypeHost && at.devicePointer != nullptr);
+}
+
+struct Shape {
+    int64_t n, kb, kpad4, nblocks, nseg, sw_bytes;
+    int narrow;
+};
+
+nvfp4_status check_shape(int64_t rows, int64_t cols, int block, Shape* sh) {
+    if (rows < 0 || cols < 0) return NVFP4_ERR_INVALID_ARG;
+    if (block != 16 && block != 32 && block != 64) return NVFP4_ERR_UNSUPPORTED;
+    if (cols % block != 0) return NVFP4_ERR_INVALID_ARG;
+    if (!mul_ok(rows, cols, &sh->n)) return NVFP4_ERR_RANGE;
+    sh->kb = cols / block;
+    sh->kpad4 = (sh->kb + 3) / 4;
+    sh->nblocks = rows * sh->kb;
+    sh->nseg = sh->n / 16;
+    int64_t rows_pad = (rows + 127) / 128 * 128, t;
+    if (!mul_ok(rows_pad, sh->kpad4 * 4, &t)) return NVFP4_ERR_RANGE;
+    sh->sw_bytes = t;
+    sh->narrow = (sh->nblocks < ((int64_t)1 << 32)) && (sh->kb < ((int64_t)1 << 32));
+    return NVFP4_OK;
+}
+
+nvfp4_status quantize_common(int method, const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                             const float* S, nvfp4_objective obj, const float* w, int64_t w_row_stride,
+                             int win_lo, int win_hi, uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled,
+                             float* block_loss, void* stream) {
+    if (dt != NVFP4_IN_BF16 && dt != NVFP4_IN_F32) return NVFP4_ERR_INVALID_ARG;
+    if (obj != NVFP4_OBJ_MSE && obj != NVFP4_OBJ_WMSE) return NVFP4_ERR_INVALID_ARG;
+    Shape sh;
+    nvfp4_status st = check_shape(rows, cols, block, &sh);
+    if (st != NVFP4_OK) return st;
+    if (sf_swizzled && block != 16) return NVFP4_ERR_UNSUPPORTED;
+    if (method == 0) {
+        if (win_lo == NVFP4_WINDOW_DEFAULT && win_hi == NVFP4_WINDOW_DEFAULT) {
+            win_lo = (obj == NVFP4_OBJ_MSE && block == 16) ? -3 : -8;   // Lemma 4.3 / Sec. 4.2.2
+            win_hi = 7;                                                 // Lemma 4.2, alpha = 12/7
+        } else if (win_lo < -126 || win_hi > 126 || win_lo > win_hi) {
+            return NVFP4_ERR_INVALID_ARG;
+        }
+    }
+    if (sh.n == 0) return NVFP4_OK;
+    if (!x || !S || !codes || (!sf_linear && !sf_swizzled)) return NVFP4_ERR_INVALID_ARG;
+    if (obj == NVFP4_OBJ_WMSE) {
+        if (!w) return NVFP4_ERR_INVALID_ARG;
+        if (w_row_stride != 0 && w_row_stride < cols) return NVFP4_ERR_INVALID_ARG;
+        if (w_row_stride < 0 || w_row_stride % 4 != 0) return NVFP4_ERR_ALIGNMENT;
+        if (!aligned(w, 16)) return NVFP4_ERR_ALIGNMENT;
+    }
+    if (!aligned(x, 16) || !aligned(codes, 8) || !aligned(S, 4) || (block_loss && !aligned(block_loss, 4)))
+        return NVFP4_ERR_ALIGNMENT;
+    const int64_t xbytes = sh.n * (dt == NVFP4_IN_BF16 ? 2 : 4);
+    int64_t wbytes = 0;
+    if (obj == NVFP4_OBJ_WMSE) {
+        if (w_row_stride == 0) {
+            wbytes = cols * 4;
+        } else if (!mul_ok(rows - 1, w_row_stride, &wbytes) || wbytes > INT64_MAX / 4 - cols) {
+            return NVFP4_ERR_RANGE;
+        } else {
+            wbytes = (wbytes + cols) * 4;
+        }
+    }
+    const int64_t cbytes = sh.n / 2, lbytes = sh.nblocks, sbytes = sh.sw_bytes, fbytes = sh.nblocks * 4;
+    const void* outs[4] = {codes, sf_linear, sf_swizzled, block_loss};
+    const int64_t olen[4] = {cbytes, lbytes, sbytes, fbytes};
+    for (int i = 0; i < 4; i++) {
+        if (!outs[i]) continue;
+        if (overlap(outs[i], olen[i], x, xbytes) || overlap(outs[i], olen[i], S, 4)) return NVFP4_ERR_INVALID_ARG;
+        if (obj == NVFP4_OBJ_WMSE && overlap(outs[i], olen[i], w, wbytes)) return NVFP4_ERR_INVALID_ARG;
+        for (int j = i + 1; j < 4; j++)
+            if (overlap(outs[i], olen[i], outs[j], olen[j])) return NVFP4_ERR_INVALID_ARG;
+    }
+    if (!device_accessible(x) || !device_accessible(S) || !device_accessible(codes) ||
+        !device_accessible(sf_linear) || !device_accessible(sf_swizzled) || !device_accessible(block_loss) ||
+        (obj == NVFP4_OBJ_WMSE && !device_accessible(w)))
+        return NVFP4_ERR_INVALID_ARG;
+    const int sms = sm_count();
+    if (sms <= 0) return NVFP4_ERR_CUDA;
+
+    QuantParams p;
+    p.x = x;
+    p.S = S;
+    p.w = (obj == NVFP4_OBJ_WMSE) ? w : nullptr;
+    p.w_row_stride = w_row_stride;
+    p.rows = rows;
+    p.cols = cols;
+    p.kb = sh.kb;
+    p.kpad4 = sh.kpad4;
+    p.nseg = sh.nseg;
+    p.narrow = sh.narrow;
+    p.win_lo = win_lo;
+    p.win_hi = win_hi;
+    p.codes = codes;
+    p.sf_linear = sf_linear;
+    p.sf_swizzled = sf_swizzled;
+    p.block_loss = block_loss;
+    cudaError_t e = launch_quantize(p, dt == NVFP4_IN_BF16 ? 0 : 1, method, obj == NVFP4_OBJ_WMSE ? 1 : 0, block,
+                                    sms, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* nvfp4_status_string(nvfp4_status st) {
+    switch (st) {
+        case NVFP4_OK: return "ok";
+        case NVFP4_ERR_INVALID_ARG: return "invalid argument";
+        case NVFP4_ERR_UNSUPPORTED: return "unsupported configuration";
+        case NVFP4_ERR_ALIGNMENT: return "misaligned pointer";
+        case NVFP4_ERR_RANGE: return "size out of range";
+        case NVFP4_ERR_CUDA: return "CUDA error";
+    }
+    return "unknown status";
+}
+
+size_t nvfp4_global_scale_workspace(int64_t n) {
+    (void)n;
+    return (size_t)kAmaxParts * (sizeof(float) + sizeof(int));
+}
+
+nvfp4_status nvfp4_global_scale(const void* x, nvfp4_dtype dt, int64_t n, float fp8_div, float* S_out,
+                                int* status_dev, void* workspace, size_t ws_bytes, void* stream) {
+    if (dt != NVFP4_IN_BF16 && dt != NVFP4_IN_F32) return NVFP4_ERR_INVALID_ARG;
+    if (n < 0 || !(fp8_div > 0.0f) || fp8_div > 1e30f) return NVFP4_ERR_INVALID_ARG;
+    if (!S_out || !workspace || (n > 0 && !x)) return NVFP4_ERR_INVALID_ARG;
+    if (ws_bytes < nvfp4_global_scale_workspace(n)) return NVFP4_ERR_INVALID_ARG;
+    if (n > INT64_MAX / 4) return NVFP4_ERR_RANGE;
+    if ((x && !aligned(x, 16)) || !aligned(workspace, 16) || !aligned(S_out, 4) ||
+        (status_dev && !aligned(status_dev, 4)))
+        return NVFP4_ERR_ALIGNMENT;
+    const int64_t xbytes = n * (dt == NVFP4_IN_BF16 ? 2 : 4);
+    if (overlap(S_out, 4, x, xbytes) || overlap(workspace, (int64_t)ws_bytes, x, xbytes) ||
+        overlap(S_out, 4, workspace, (int64_t)ws_bytes) || overlap(status_dev, 4, S_out, 4) ||
+        overlap(status_dev, 4, workspace, (int64_t)ws_bytes) || overlap(status_dev, 4, x, xbytes))
+        return NVFP4_ERR_INVALID_ARG;
+    if (!device_accessible(x) || !device_accessible(S_out) || !device_accessible(workspace) ||
+        !device_accessible(status_dev))
+        return NVFP4_ERR_INVALID_ARG;
+    const int sms = sm_count();
+    if (sms <= 0) return NVFP4_ERR_CUDA;
+    cudaError_t e = launch_global_scale(x, dt == NVFP4_IN_BF16 ? 0 : 1, n, fp8_div, S_out, status_dev, workspace, sms,
+                                        static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
+}
+
+nvfp4_status scalesweep_quantize(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                                 const float* S, nvfp4_objective obj, const float* w, int64_t w_row_stride,
+                                 int win_lo, int win_hi, uint8_t* codes, uint8_t* sf_linear,
+                                 uint8_t* sf_swizzled, float* block_loss, void* stream) {
+    return quantize_common(0, x, dt, rows, cols, block, S, obj, w, w_row_stride, win_lo, win_hi, codes, sf_linear,
+                           sf_swizzled, block_loss, stream);
+}
+
+nvfp4_status absmax_quantize(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                             const float* S, uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled,
+                             float* block_loss, void* stream) {
+    return quantize_common(1, x, dt, rows, cols, block, S, NVFP4_OBJ_MSE, nullptr, 0, 0, 0, codes, sf_linear,
+                           sf_swizzled, block_loss, stream);
+}
+
+nvfp4_status four_over_six_quantize(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                                    const float* S, nvfp4_objective obj, const float* w, int64_t w_row_stride,
+                                    uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled,
+                                    float* block_loss, void* stream) {
+    return quantize_common(2, x, dt, rows, cols, block, S, obj, w, w_row_stride, 0, 0, codes, sf_linear, sf_swizzled,
+                           block_loss, stream);
+}
+
+nvfp4_status nvfp4_dequantize(const uint8_t* codes, const uint8_t* sf, nvfp4_sf_layout layout, const float* S,
+                              int64_t rows, int64_t cols, int block, void* out, nvfp4_dtype out_dt,
+                              void* stream) {
+    if (layout != NVFP4_SF_LINEAR && layout != NVFP4_SF_SWIZZLED) return NVFP4_ERR_INVALID_ARG;
+    if (out_dt != NVFP4_IN_BF16 && out_dt != NVFP4_IN_F32) return NVFP4_ERR_INVALID_ARG;
+    Shape sh;
+    nvfp4_status st = check_shape(rows, cols, block, &sh);
+    if (st != NVFP4_OK) return st;
+    if (layout == NVFP4_SF_SWIZZLED && block != 16) return NVFP4_ERR_UNSUPPORTED;
+    if (sh.n == 0) return NVFP4_OK;
+    if (!codes || !sf || !S || !out) return NVFP4_ERR_INVALID_ARG;
+    if (!aligned(codes, 8) || !aligned(out, 16) || !aligned(S, 4)) return NVFP4_ERR_ALIGNMENT;
+    const int64_t obytes = sh.n * (out_dt == NVFP4_IN_BF16 ? 2 : 4);
+    const int64_t sfbytes = layout == NVFP4_SF_SWIZZLED ? sh.sw_bytes : sh.nblocks;
+    if (overlap(out, obytes, codes, sh.n / 2) || overlap(out, obytes, sf, sfbytes) || overlap(out, obytes, S, 4))
+        return NVFP4_ERR_INVALID_ARG;
+    if (!device_accessible(codes) || !device_accessible(sf) || !device_accessible(S) || !device_accessible(out))
+        return NVFP4_ERR_INVALID_ARG;
+    const int sms = sm_count();
+    if (sms <= 0) return NVFP4_ERR_CUDA;
+    DequantParams p;
+    p.codes = codes;
+    p.sf = sf;
+    p.S = S;
+    p.rows = rows;
+    p.cols = cols;
+    p.kb = sh.kb;
+    p.kpad4 = sh.kpad4;
+    p.nseg = sh.nseg;
+    p.narrow = sh.narrow;
+    p.swizzled = layout == NVFP4_SF_SWIZZLED;
+    p.block = block;
+    p.out = out;
+    cudaError_t e = launch_dequantize(p, out_dt == NVFP4_IN_BF16 ? 0 : 1, sms, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
+}
+
+}  // extern "C"

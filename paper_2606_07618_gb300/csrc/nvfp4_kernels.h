@@ -1,0 +1,46 @@
+// Internal interface between the C-ABI host layer (api.cu) and the kernel
+// translation units.  Not part of the public ABI.
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace nvfp4 {
+
+struct QuantParams {
+    const void* x;
+    const float* S;
+    const float* w;
+    int64_t w_row_stride;
+    int64_t rows, cols, kb, kpad4;
+    int64_t nseg;            // rows * cols / 16
+    int narrow;              // rows * kb < 2^32
+    int win_lo, win_hi;
+    uint8_t* codes;
+    uint8_t* sf_linear;
+    uint8_t* sf_swizzled;
+    float* block_loss;
+};
+
+// dtype 0 bf16 / 1 f32; method 0 ScaleSweep / 1 AbsMax / 2 four-over-six;
+// obj 0 MSE / 1 WMSE; block 16/32/64; sms = multiprocessor count.
+cudaError_t launch_quantize(const QuantParams& p, int dtype, int method, int obj, int block, int sms,
+                            cudaStream_t s);
+
+// Global-scale reduction: partial maxima into ws, then S and the status word.
+cudaError_t launch_global_scale(const void* x, int dtype, int64_t n, float fp8_div, float* S_out,
+                                int* status_dev, void* ws, int sms, cudaStream_t s);
+constexpr int kAmaxParts = 1024;   // partial slots in the workspace
+
+struct DequantParams {
+    const uint8_t* codes;
+    const uint8_t* sf;
+    const float* S;
+    int64_t rows, cols, kb, kpad4, nseg;
+    int narrow;
+    int swizzled;
+    int block;
+    void* out;
+};
+cudaError_t launch_dequantize(const DequantParams& p, int out_dtype, int sms, cudaStream_t s);
+
+}  // namespace nvfp4

@@ -1,0 +1,194 @@
+// Global scale S = amax / (6 D) (Sec. 3.2 with D = 448; Sec. 4.2.1 with D = 256)
+// and NVFP4 dequantisation x_hat = q * s * S (Sec. 3.2).
+//
+// amax is a two-launch reduction: a persistent grid of streaming 16-byte loads
+// writes one partial maximum (and a NaN/inf flag) per CTA into the caller's
+// workspace, then a single CTA folds the partials and writes S on the device.
+// No atomics and no zero-initialised state, so back-to-back calls on one
+// workspace need nothing in between.  Max is exact, so the order is free.
+#include <cuda_bf16.h>
+
+#include "nvfp4_device.cuh"
+#include "nvfp4_kernels.h"
+
+namespace nvfp4 {
+
+__device__ __forceinline__ void amax_acc(float v, float& m, int& bad) {
+    if (!isfinite(v)) bad = 1;
+    m = fmaxf(m, fabsf(v));                  // fmaxf drops NaN, keeps inf
+}
+
+template <int DT>
+__global__ void __launch_bounds__(256) amax_partial_kernel(const void* x, int64_t n, float* part_max,
+                                                           int* part_bad) {
+    constexpr int PER = DT == 0 ? 8 : 4;      // elements per 16-byte vector
+    const int64_t nvec = n / PER;
+    float m = 0.0f;
+    int bad = 0;
+    const uint4* xv = static_cast<const uint4*>(x);
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += stride) {
+        uint4 u = ld_stream16(xv + i);
+        uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            if (DT == 0) {
+                amax_acc(bf16lo(w[j]), m, bad);
+                amax_acc(bf16hi(w[j]), m, bad);
+            } else {
+                amax_acc(__uint_as_float(w[j]), m, bad);
+            }
+        }
+    }
+    // tail elements (n not a multiple of the vector width)
+    if (blockIdx.x == 0 && threadIdx.x < (int)(n - nvec * PER)) {
+        const int64_t i = nvec * PER + threadIdx.x;
+        float v = DT == 0 ? __uint_as_float((uint32_t)(static_cast<const uint16_t*>(x)[i]) << 16)
+                          : static_cast<const float*>(x)[i];
+        amax_acc(v, m, bad);
+    }
+    // non-negative floats order like their bit patterns
+    uint32_t mb = __reduce_max_sync(0xffffffffu, __float_as_uint(m));
+    int anybad = __reduce_or_sync(0xffffffffu, (unsigned)bad);
+    __shared__ uint32_t sm[8];
+    __shared__ int sb[8];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        sm[warp] = mb;
+        sb[warp] = anybad;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        uint32_t v = lane < (int)(blockDim.x >> 5) ? sm[lane] : 0u;
+        int b = lane < (int)(blockDim.x >> 5) ? sb[lane] : 0;
+        v = __reduce_max_sync(0xffffffffu, v);
+        b = __reduce_or_sync(0xffffffffu, (unsigned)b);
+        if (lane == 0) {
+            part_max[blockIdx.x] = __uint_as_float(v);
+            part_bad[blockIdx.x] = b;
+        }
+    }
+}
+
+__global__ void __launch_bounds__(256) amax_final_kernel(const float* part_max, const int* part_bad, int nparts,
+                                                         float fp8_div, float* S_out, int* status_dev) {
+    uint32_t v = 0u;
+    int b = 0;
+    for (int i = threadIdx.x; i < nparts; i += blockDim.x) {
+        v = max(v, __float_as_uint(part_max[i]));
+        b |= part_bad[i];
+    }
+    v = __reduce_max_sync(0xffffffffu, v);
+    b = __reduce_or_sync(0xffffffffu, (unsigned)b);
+    __shared__ uint32_t sm[8];
+    __shared__ int sb[8];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        sm[warp] = v;
+        sb[warp] = b;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t m = 0;
+        int bad = 0;
+        for (int i = 0; i < (int)(blockDim.x >> 5); i++) {
+            m = max(m, sm[i]);
+            bad |= sb[i];
+        }
+        const float amax = __uint_as_float(m);
+        S_out[0] = __fdiv_rn(amax, __fmul_rn(6.0f, fp8_div));
+        if (status_dev && bad) atomicOr(status_dev, 1);
+    }
+}
+
+cudaError_t launch_global_scale(const void* x, int dtype, int64_t n, float fp8_div, float* S_out,
+                                int* status_dev, void* ws, int sms, cudaStream_t s) {
+    float* part_max = static_cast<float*>(ws);
+    int* part_bad = reinterpret_cast<int*>(part_max + kAmaxParts);
+    const int per = dtype == 0 ? 8 : 4;
+    const int64_t nvec = n / per;
+    int64_t grid = (nvec + 255) / 256;
+    if (grid > (int64_t)sms * 4) grid = (int64_t)sms * 4;
+    if (grid > kAmaxParts) grid = kAmaxParts;
+    if (grid < 1) grid = 1;
+    if (dtype == 0)
+        amax_partial_kernel<0><<<(int)grid, 256, 0, s>>>(x, n, part_max, part_bad);
+    else
+        amax_partial_kernel<1><<<(int)grid, 256, 0, s>>>(x, n, part_max, part_bad);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    amax_final_kernel<<<1, 256, 0, s>>>(part_max, part_bad, (int)grid, fp8_div, S_out, status_dev);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Dequantisation: one thread per 16-element segment.  q and s are decoded by
+// the native converts into f16, q*s is exact in f16 (at most 7 significant
+// bits, within range), then one fp32 multiply by S rounds once.
+template <int OUT_BF16>
+__global__ void __launch_bounds__(256) dequant_kernel(DequantParams p) {
+    const float S = __ldg(p.S);
+    const int segs = p.block / 16;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < p.nseg; g += stride) {
+        const int64_t blk = g / segs;
+        int64_t so = blk;
+        if (p.swizzled) {
+            int64_t row, kbi;
+            if (p.narrow) {
+                const uint32_t b32 = (uint32_t)blk, k32 = (uint32_t)p.kb, r32 = b32 / k32;
+                row = r32;
+                kbi = b32 - r32 * k32;
+            } else {
+                row = blk / p.kb;
+                kbi = blk - row * p.kb;
+            }
+            so = swizzle_offset(row, kbi, p.kpad4);
+        }
+        const uint16_t vh = e4m3_to_f16bits(p.sf[so]);
+        const uint32_t vv = (uint32_t)vh * 0x10001u;
+        const uint2 c = *reinterpret_cast<const uint2*>(p.codes + g * 8);
+        const uint32_t cw[2] = {c.x, c.y};
+        float out[16];
+#pragma unroll
+        for (int h = 0; h < 2; h++) {
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                uint32_t q2, prod;
+                const uint16_t byte = (uint16_t)((cw[h] >> (8 * j)) & 0xFFu);
+                asm("{\n\t.reg .b8 b;\n\tcvt.u8.u16 b, %1;\n\tcvt.rn.f16x2.e2m1x2 %0, b;\n\t}" : "=r"(q2) : "h"(byte));
+                asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(prod) : "r"(q2), "r"(vv));
+                out[8 * h + 2 * j] = __fmul_rn(f16bits_to_f32((uint16_t)(prod & 0xFFFF)), S);
+                out[8 * h + 2 * j + 1] = __fmul_rn(f16bits_to_f32((uint16_t)(prod >> 16)), S);
+            }
+        }
+        if (OUT_BF16) {
+            uint32_t o[8];
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                __nv_bfloat16 a = __float2bfloat16_rn(out[2 * j]), b = __float2bfloat16_rn(out[2 * j + 1]);
+                o[j] = (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(b) << 16);
+            }
+            uint4* op = reinterpret_cast<uint4*>(static_cast<char*>(p.out) + g * 32);
+            op[0] = make_uint4(o[0], o[1], o[2], o[3]);
+            op[1] = make_uint4(o[4], o[5], o[6], o[7]);
+        } else {
+            float4* op = reinterpret_cast<float4*>(static_cast<char*>(p.out) + g * 64);
+#pragma unroll
+            for (int j = 0; j < 4; j++) op[j] = make_float4(out[4 * j], out[4 * j + 1], out[4 * j + 2], out[4 * j + 3]);
+        }
+    }
+}
+
+cudaError_t launch_dequantize(const DequantParams& p, int out_dtype, int sms, cudaStream_t s) {
+    if (p.nseg <= 0) return cudaSuccess;
+    int64_t grid = (p.nseg + 255) / 256;
+    if (grid > (int64_t)sms * 8) grid = (int64_t)sms * 8;
+    if (out_dtype == 0)
+        dequant_kernel<1><<<(int)grid, 256, 0, s>>>(p);
+    else
+        dequant_kernel<0><<<(int)grid, 256, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace nvfp4

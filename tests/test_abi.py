@@ -1,0 +1,80 @@
+"""The C-ABI library builds, loads and exports every entry point declared in
+include/nvfp4ss.h; argument validation happens on the host before any CUDA
+call, so it is exercised here without a GPU (no compute call is made)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from conftest import ROOT
+
+HEADER = os.path.join(ROOT, "include", "nvfp4ss.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\**\s+([a-z0-9_]+)\s*\(", src, re.M)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2606_07618_gb300 import binding
+    return binding.lib()
+
+
+def test_header_declares_the_api():
+    assert declared_functions() == sorted([
+        "nvfp4_status_string", "nvfp4_global_scale_workspace", "nvfp4_global_scale", "scalesweep_quantize",
+        "absmax_quantize", "four_over_six_quantize", "nvfp4_dequantize"])
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in declared_functions():
+        assert hasattr(L, name), name
+
+
+def test_status_strings(L):
+    from paper_2606_07618_gb300 import binding
+    assert binding.nvfp4_status_string(0) == "ok"
+    assert binding.nvfp4_status_string(3) == "misaligned pointer"
+    assert binding.nvfp4_global_scale_workspace(1 << 30) >= 8
+
+
+FAKE = 0x10000000  # never dereferenced: every call below fails validation first
+
+
+def _ss(L, x=FAKE, dt=0, rows=4, cols=64, block=16, S=FAKE, obj=0, w=None, stride=0, lo=-(2 ** 31), hi=-(2 ** 31),
+        codes=FAKE + 0x100000, sfl=FAKE + 0x200000, sfs=None, loss=None):
+    return L.scalesweep_quantize(x, dt, rows, cols, block, S, obj, w, stride, lo, hi, codes, sfl, sfs, loss, None)
+
+
+def test_validation_without_gpu(L):
+    assert _ss(L, block=8) == 2                       # unsupported block
+    assert _ss(L, block=32, sfs=FAKE + 0x300000) == 2  # swizzled needs block 16
+    assert _ss(L, cols=40) == 1                       # cols % block
+    assert _ss(L, rows=-1) == 1
+    assert _ss(L, dt=7) == 1
+    assert _ss(L, obj=3) == 1
+    assert _ss(L, lo=-3, hi=-4) == 1                  # empty window
+    assert _ss(L, lo=-127, hi=7) == 1
+    assert _ss(L, lo=-(2 ** 31), hi=7) == 1           # half-default window
+    assert _ss(L, rows=0) == 0                        # empty input: nothing to do, no launch
+    assert _ss(L, x=None) == 1
+    assert _ss(L, sfl=None) == 1                      # no scale output at all
+    assert _ss(L, obj=1, w=None) == 1                 # WMSE needs weights
+    assert _ss(L, obj=1, w=FAKE + 0x400000, stride=8) == 1  # stride shorter than a row
+    assert _ss(L, x=FAKE + 2) == 3                    # misaligned input
+    assert _ss(L, codes=FAKE + 0x100004) == 3         # misaligned codes
+    assert _ss(L, obj=1, w=FAKE + 0x400004) == 3      # misaligned weights
+    assert _ss(L, codes=FAKE) == 1                    # output overlaps input
+    assert _ss(L, sfl=FAKE + 0x100010) == 1           # outputs overlap each other
+    assert _ss(L, rows=2 ** 40, cols=2 ** 40) == 4    # size overflow
+    assert L.nvfp4_global_scale(FAKE, 0, 100, ctypes.c_float(0.0), FAKE + 4096, None, FAKE + 8192, 1 << 20, None) == 1
+    assert L.nvfp4_global_scale(FAKE + 2, 0, 100, ctypes.c_float(256.0), FAKE + 4096, None, FAKE + 8192, 1 << 20,
+                                None) == 3
+    assert L.nvfp4_global_scale(FAKE, 0, 100, ctypes.c_float(256.0), FAKE + 4096, None, FAKE + 8192, 16, None) == 1
+    assert L.nvfp4_dequantize(FAKE, FAKE + 4096, 2, FAKE + 8192, 4, 64, 32, FAKE + 16384, 1, None) == 2
+    assert L.nvfp4_dequantize(FAKE, FAKE + 4096, 3, FAKE + 8192, 4, 64, 16, FAKE + 16384, 1, None) == 1
+    assert L.nvfp4_dequantize(FAKE, FAKE + 4096, 1, FAKE + 8192, 4, 64, 16, FAKE + 8, 1, None) == 3

@@ -173,6 +173,8 @@ def test_scalesweep_dominates_absmax_and_four_six(oracle_mod, block, objective):
         # the recorded AbsMax loss is the loss of its own scale codes
         Lam = oracle_mod.block_losses_at(x, block, S, am["sf"], objective, w=w)
         assert np.array_equal(Lam, am["best"])
+        Lss, css = oracle_mod.block_losses_at(x, block, S, ss["sf"], objective, w=w, want_codes=True)
+        assert np.array_equal(Lss, ss["best"]) and np.array_equal(css, ss["codes"])
 
 
 def test_lemma1_halving_in_oracle_arithmetic(oracle_mod):
