@@ -87,6 +87,28 @@ nvfp4_status nvfp4_global_scale(const void* x, nvfp4_dtype dt, int64_t n, float 
                                 int* status_dev, void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * nvfp4_global_scale without a workspace argument; the paper has no
+ * counterpart (it is a packaging variant of the reduction above).
+ * For callers that cannot call cudaMalloc: code that runs under a device-memory
+ * plan fixed at start-up (e.g. a serving engine that reserves all GPU memory
+ * up front and forbids allocation on the request path) or a host embedding
+ * this library without an allocator of its own, and so cannot provide the
+ * workspace nvfp4_global_scale needs.  The scratch is a 128 KiB static device
+ * array that every GPU which loads the library holds until the process exits;
+ * no allocation or free is made by any call.
+ *   Same S, status word and alignment rules as nvfp4_global_scale.
+ *   n may be at most 2^29 bf16 or 2^28 fp32 elements; a larger n returns
+ *   NVFP4_ERR_RANGE and launches nothing.
+ *   The first call on each device looks up the scratch's device address
+ *   (cudaGetSymbolAddress) once, with that device current; make that first call
+ *   before any stream capture.
+ *   All calls share the one scratch array: calls whose kernels may overlap on
+ *   the GPU (e.g. on unordered streams) race and must be ordered by the caller.
+ */
+nvfp4_status nvfp4_global_scale_noalloc(const void* x, nvfp4_dtype dt, int64_t n, float fp8_div, float* S_out,
+                                        int* status_dev, void* stream);
+
+/*
  * ScaleSweep quantisation (Sec. 4.2.2): per block, sweep the E4M3 scale codes
  * in [I0 + win_lo, I0 + win_hi] (clamped to 1..126), score each with the MSE
  * (Sec. 4.1, Eq. for L^MSE) or WMSE (Sec. 4.1, diagonal-Gram importance)

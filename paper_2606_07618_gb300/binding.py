@@ -50,12 +50,13 @@ def lib() -> ctypes.CDLL:
         L.nvfp4_status_string.argtypes, L.nvfp4_status_string.restype = [i], ctypes.c_char_p
         L.nvfp4_global_scale_workspace.argtypes, L.nvfp4_global_scale_workspace.restype = [i64], sz
         L.nvfp4_global_scale.argtypes = [p, i, i64, f, p, p, p, sz, p]
+        L.nvfp4_global_scale_noalloc.argtypes = [p, i, i64, f, p, p, p]
         L.scalesweep_quantize.argtypes = [p, i, i64, i64, i, p, i, p, i64, i, i, p, p, p, p, p]
         L.absmax_quantize.argtypes = [p, i, i64, i64, i, p, p, p, p, p, p]
         L.four_over_six_quantize.argtypes = [p, i, i64, i64, i, p, i, p, i64, p, p, p, p, p]
         L.nvfp4_dequantize.argtypes = [p, p, i, p, i64, i64, i, p, i, p]
-        for fn in ("nvfp4_global_scale", "scalesweep_quantize", "absmax_quantize", "four_over_six_quantize",
-                   "nvfp4_dequantize"):
+        for fn in ("nvfp4_global_scale", "nvfp4_global_scale_noalloc", "scalesweep_quantize", "absmax_quantize",
+                   "four_over_six_quantize", "nvfp4_dequantize"):
             getattr(L, fn).restype = i
         _lib = L
     return _lib
@@ -103,6 +104,14 @@ def nvfp4_global_scale(x, fp8_div: float, S_out, status=None, workspace=None, st
     rc = lib().nvfp4_global_scale(_ptr(x), _dtype(x), x.numel(), float(fp8_div), _ptr(S_out), _ptr(status),
                                   _ptr(workspace), ws_bytes, _stream(stream))
     _check("nvfp4_global_scale", rc)
+
+
+def nvfp4_global_scale_noalloc(x, fp8_div: float, S_out, status=None, stream=None):
+    """Global scale for callers that cannot allocate: no workspace argument
+    (the library's static device scratch is used instead)."""
+    rc = lib().nvfp4_global_scale_noalloc(_ptr(x), _dtype(x), x.numel(), float(fp8_div), _ptr(S_out), _ptr(status),
+                                          _stream(stream))
+    _check("nvfp4_global_scale_noalloc", rc)
 
 
 def scalesweep_quantize(x, block: int, S, objective: int, w, w_row_stride: int, win_lo: int, win_hi: int,

@@ -31,6 +31,10 @@ cudaError_t launch_global_scale(const void* x, int dtype, int64_t n, float fp8_d
                                 int* status_dev, void* ws, int sms, cudaStream_t s);
 constexpr int kAmaxParts = 1024;   // partial slots in the workspace
 
+// Same two kernels with caller-chosen partial slots and grid (grid <= slots).
+cudaError_t launch_global_scale_parts(const void* x, int dtype, int64_t n, float fp8_div, float* S_out,
+                                      int* status_dev, float* part_max, int* part_bad, int grid, cudaStream_t s);
+
 struct DequantParams {
     const uint8_t* codes;
     const uint8_t* sf;

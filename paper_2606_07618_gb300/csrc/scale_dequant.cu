@@ -121,6 +121,18 @@ cudaError_t launch_global_scale(const void* x, int dtype, int64_t n, float fp8_d
     return cudaGetLastError();
 }
 
+cudaError_t launch_global_scale_parts(const void* x, int dtype, int64_t n, float fp8_div, float* S_out,
+                                      int* status_dev, float* part_max, int* part_bad, int grid, cudaStream_t s) {
+    if (dtype == 0)
+        amax_partial_kernel<0><<<grid, 256, 0, s>>>(x, n, part_max, part_bad);
+    else
+        amax_partial_kernel<1><<<grid, 256, 0, s>>>(x, n, part_max, part_bad);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    amax_final_kernel<<<1, 256, 0, s>>>(part_max, part_bad, grid, fp8_div, S_out, status_dev);
+    return cudaGetLastError();
+}
+
 // ---------------------------------------------------------------------------
 // Dequantisation: one thread per 16-element segment.  q and s are decoded by
 // the native converts into f16, q*s is exact in f16 (at most 7 significant
