@@ -411,6 +411,49 @@ def config_dict(wl, world):
             "l2": "no flush: each step streams 436 MB of inputs (> 129 MB L2); sweeps run after all 7 amax passes"}
 
 
+def run_kernel_case(args):
+    """One kernel on one synthetic [rows, cols] tensor (larger than L2 by
+    default), timed with CUDA events; used for ncu captures and sweeps."""
+    from paper_2606_07618_gb300 import binding as B
+    from paper_2606_07618_gb300 import workloads as W
+    dev = "cuda"
+    x = W.small_tensor(args.rows, args.cols, 7, dist="normal", std=0.02, outliers=max(1, args.cols // 1000),
+                       mult=20.0).to(dev)
+    w = torch.exp(torch.randn(args.cols, generator=torch.Generator().manual_seed(3))).to(dev)
+    S = torch.empty(1, device=dev)
+    ws = torch.empty(B.nvfp4_global_scale_workspace(x.numel()), dtype=torch.uint8, device=dev)
+    B.nvfp4_global_scale(x, 256.0, S, None, ws)
+    o = B.empty_outputs(args.rows, args.cols, args.block, device=dev, linear=True, swizzled=args.block == 16)
+    win = (B.NVFP4_WINDOW_DEFAULT, B.NVFP4_WINDOW_DEFAULT)
+    dq = torch.empty(args.rows, args.cols, dtype=torch.bfloat16, device=dev)
+    fns = {
+        "sweep_wmse": lambda: B.scalesweep_quantize(x, args.block, S, 1, w, 0, *win, o["codes"], o["sf_linear"],
+                                                    o["sf_swizzled"]),
+        "sweep_mse": lambda: B.scalesweep_quantize(x, args.block, S, 0, None, 0, *win, o["codes"], o["sf_linear"],
+                                                   o["sf_swizzled"]),
+        "absmax": lambda: B.absmax_quantize(x, args.block, S, o["codes"], o["sf_linear"], o["sf_swizzled"]),
+        "four_six": lambda: B.four_over_six_quantize(x, args.block, S, 1, w, 0, o["codes"], o["sf_linear"],
+                                                     o["sf_swizzled"]),
+        "dequant": lambda: B.nvfp4_dequantize(o["codes"], o["sf_linear"], 1, S, args.rows, args.cols, args.block, dq),
+        "amax": lambda: B.nvfp4_global_scale(x, 256.0, S, None, ws),
+    }
+    fn = fns[args.kernel_case]
+    fns["sweep_mse"]()
+    for _ in range(2):
+        fn()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(args.reps):
+        fn()
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / args.reps
+    n = x.numel()
+    print(json.dumps({"kernel_case": args.kernel_case, "rows": args.rows, "cols": args.cols, "block": args.block,
+                      "ms": round(ms, 4), "gelem_s": round(n / ms / 1e6, 2)}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -421,7 +464,16 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-rows", type=int, default=64)
+    ap.add_argument("--kernel-case", default=None,
+                    choices=["sweep_wmse", "sweep_mse", "absmax", "four_six", "dequant", "amax"])
+    ap.add_argument("--rows", type=int, default=16384)
+    ap.add_argument("--cols", type=int, default=8192)
+    ap.add_argument("--block", type=int, default=16)
+    ap.add_argument("--reps", type=int, default=5)
     args = ap.parse_args()
+    if args.kernel_case:
+        run_kernel_case(args)
+        return
     if args.warmup < 3:
         args.warmup = 3
 

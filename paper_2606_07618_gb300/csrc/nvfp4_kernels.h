@@ -6,6 +6,11 @@
 
 namespace nvfp4 {
 
+struct FastDiv {            // n / d = (t + ((n - t) >> s1)) >> s2, t = umulhi(n, mul)
+    uint32_t mul, s1, s2;
+};
+FastDiv make_fast_div(uint32_t d);
+
 struct QuantParams {
     const void* x;
     const float* S;
@@ -14,6 +19,8 @@ struct QuantParams {
     int64_t rows, cols, kb, kpad4;
     int64_t nseg;            // rows * cols / 16
     int narrow;              // rows * kb < 2^32
+    int need_rowcol;         // swizzled scales or weights need (row, block column)
+    FastDiv kb_div;          // divides a 32-bit block index by kb
     int win_lo, win_hi;
     uint8_t* codes;
     uint8_t* sf_linear;

@@ -27,9 +27,8 @@ __global__ void __launch_bounds__(256) amax_partial_kernel(const void* x, int64_
     int bad = 0;
     const uint4* xv = static_cast<const uint4*>(x);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += stride) {
-        uint4 u = ld_stream16(xv + i);
-        uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    auto fold = [&](const uint4& u) {
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
         for (int j = 0; j < 4; j++) {
             if (DT == 0) {
@@ -39,7 +38,18 @@ __global__ void __launch_bounds__(256) amax_partial_kernel(const void* x, int64_
                 amax_acc(__uint_as_float(w[j]), m, bad);
             }
         }
+    };
+    int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    // four independent 16-byte loads in flight per thread
+    for (; i + 3 * stride < nvec; i += 4 * stride) {
+        const uint4 u0 = ld_stream16(xv + i), u1 = ld_stream16(xv + i + stride);
+        const uint4 u2 = ld_stream16(xv + i + 2 * stride), u3 = ld_stream16(xv + i + 3 * stride);
+        fold(u0);
+        fold(u1);
+        fold(u2);
+        fold(u3);
     }
+    for (; i < nvec; i += stride) fold(ld_stream16(xv + i));
     // tail elements (n not a multiple of the vector width)
     if (blockIdx.x == 0 && threadIdx.x < (int)(n - nvec * PER)) {
         const int64_t i = nvec * PER + threadIdx.x;
@@ -142,24 +152,36 @@ __global__ void __launch_bounds__(256) dequant_kernel(DequantParams p) {
     const float S = __ldg(p.S);
     const int segs = p.block / 16;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < p.nseg; g += stride) {
+    auto scale_offset = [&](int64_t g) -> int64_t {
         const int64_t blk = g / segs;
-        int64_t so = blk;
-        if (p.swizzled) {
-            int64_t row, kbi;
-            if (p.narrow) {
-                const uint32_t b32 = (uint32_t)blk, k32 = (uint32_t)p.kb, r32 = b32 / k32;
-                row = r32;
-                kbi = b32 - r32 * k32;
-            } else {
-                row = blk / p.kb;
-                kbi = blk - row * p.kb;
-            }
-            so = swizzle_offset(row, kbi, p.kpad4);
+        if (!p.swizzled) return blk;
+        int64_t row, kbi;
+        if (p.narrow) {
+            const uint32_t b32 = (uint32_t)blk, k32 = (uint32_t)p.kb, r32 = b32 / k32;
+            row = r32;
+            kbi = b32 - r32 * k32;
+        } else {
+            row = blk / p.kb;
+            kbi = blk - row * p.kb;
         }
-        const uint16_t vh = e4m3_to_f16bits(p.sf[so]);
+        return swizzle_offset(row, kbi, p.kpad4);
+    };
+    int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    uint2 c_next = make_uint2(0, 0);
+    uint8_t s_next = 0;
+    if (g < p.nseg) {
+        c_next = __ldg(reinterpret_cast<const uint2*>(p.codes + g * 8));
+        s_next = __ldg(p.sf + scale_offset(g));
+    }
+    for (; g < p.nseg; g += stride) {
+        const uint2 c = c_next;
+        const uint8_t sc = s_next;
+        if (g + stride < p.nseg) {                 // prefetch the next segment
+            c_next = __ldg(reinterpret_cast<const uint2*>(p.codes + (g + stride) * 8));
+            s_next = __ldg(p.sf + scale_offset(g + stride));
+        }
+        const uint16_t vh = e4m3_to_f16bits(sc);
         const uint32_t vv = (uint32_t)vh * 0x10001u;
-        const uint2 c = *reinterpret_cast<const uint2*>(p.codes + g * 8);
         const uint32_t cw[2] = {c.x, c.y};
         float out[16];
 #pragma unroll

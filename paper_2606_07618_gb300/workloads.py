@@ -146,7 +146,8 @@ def draw(t: Tensor, rows: slice | None = None) -> torch.Tensor:
             chi.add_(n * n)
         x = z / torch.sqrt(chi / 3.0)
     elif t.dist == "laplace":
-        u = torch.rand(R, C, generator=g, dtype=torch.float32).sub_(0.5)
+        # u uniform on the open interval (-1/2, 1/2): rand() can return 0, which would give ln(0)
+        u = torch.rand(R, C, generator=g, dtype=torch.float32).clamp_(min=2.0 ** -25).sub_(0.5)
         x = u.abs().mul_(-2.0).log1p_().mul_(-t.std)
         x.mul_(torch.sign(u))
         del u
