@@ -133,6 +133,35 @@ def make_inputs(device: str):
     return wl, xs, ws
 
 
+def sweep_traffic_per_launch(elems_per_launch):
+    """DRAM bytes per sweep launch from the committed ncu capture
+    (profiles/quantize_kernel_wmse_traffic.json), scaled by elements; None if
+    the kernel sources changed since the capture."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "quantize_kernel_wmse_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+        h = hashlib.sha256()
+        for fn in rec["source_files"]:
+            with open(os.path.join(ROOT, fn), "rb") as f:
+                h.update(f.read())
+        if h.hexdigest() != rec["source_sha256"]:
+            return None
+        return round(rec["dram_bytes_per_element"] * elems_per_launch)
+    except (OSError, KeyError, ValueError):
+        return None
+
+
+def reduce_max_ms(ms: float, world: int, device) -> float:
+    """Slowest rank's time (the whole-job time under weak scaling)."""
+    if world <= 1:
+        return ms
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
 def alg_bytes_per_elem(block=16, in_bytes=2, both_layouts=True):
     return in_bytes + 0.5 + (1.0 / block) * (2 if both_layouts else 1)
 
@@ -196,10 +225,7 @@ def run_gpu(args, rank, world):
         torch.distributed.barrier()
     ms = t0.elapsed_time(t1)
     sweep_ms = sum(ev[k][i][0].elapsed_time(ev[k][i][1]) for k in range(args.steps) for i in range(len(xs)))
-    if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = reduce_max_ms(ms, world, dev)
     ms_step = ms / args.steps
     value = world * total / (ms_step * 1e-3) / 1e9
 
@@ -228,15 +254,7 @@ def run_gpu(args, rank, world):
                 "hbm": {"achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s", "frac": round(gbs / hbm_peak, 4),
                         "peak_kind": peak_kind, "bytes_per_elem": bpe},
                 "sweep_ms_per_step": round(sweep_s_per_step * 1e3, 4)}
-    traffic_file = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(traffic_file):
-        try:
-            with open(traffic_file) as f:
-                tr = json.load(f).get("scalesweep_wmse_bf16_b16")
-            if tr:
-                roofline["traffic"] = tr
-        except (OSError, ValueError):
-            pass
+    roofline["traffic"] = sweep_traffic_per_launch(total / len(xs))
 
     # ---- overhead vs the AbsMax kernel on the same tensors, same S and layouts
     def time_leg(fn, reps):
@@ -308,24 +326,54 @@ def run_gpu(args, rank, world):
         hsfl = [torch.empty_like(o["sf_linear"], device="cpu").pin_memory() for o in outs]
         hsfs = [torch.empty_like(o["sf_swizzled"], device="cpu").pin_memory() for o in outs]
         dx = [torch.empty_like(x) for x in xs]
+        eouts = [B.empty_outputs(x.shape[0], x.shape[1], 16, device=dev, linear=True, swizzled=True) for x in xs]
+        up, down = torch.cuda.Stream(), torch.cuda.Stream()
+        S2 = torch.empty(len(xs), dtype=torch.float32, device=dev)
+        wsp2 = torch.empty_like(wsp)
 
         def e2e_step():
+            # three streams: H2D of tensor i+1 and D2H of tensor i-1 overlap the
+            # kernels of tensor i; events order each tensor's copy -> compute -> copy
+            loaded, done = [], []
+            up.wait_stream(stream)          # the previous step's kernels are done with dx
             for i in range(len(xs)):
-                dx[i].copy_(hx[i], non_blocking=True)
-                B.nvfp4_global_scale(dx[i], D, S[i:i + 1], st, wsp, stream=stream)
-                o = outs[i]
-                B.scalesweep_quantize(dx[i], 16, S[i:i + 1], B.NVFP4_OBJ_WMSE, ws[i], 0, *win, o["codes"],
+                with torch.cuda.stream(up):
+                    dx[i].copy_(hx[i], non_blocking=True)
+                    ev = torch.cuda.Event()
+                    ev.record(up)
+                    loaded.append(ev)
+            for i in range(len(xs)):
+                stream.wait_event(loaded[i])
+                o = eouts[i]
+                B.nvfp4_global_scale(dx[i], D, S2[i:i + 1], st, wsp2, stream=stream)
+                B.scalesweep_quantize(dx[i], 16, S2[i:i + 1], B.NVFP4_OBJ_WMSE, ws[i], 0, *win, o["codes"],
                                       o["sf_linear"], o["sf_swizzled"], None, stream=stream)
-                hcodes[i].copy_(o["codes"], non_blocking=True)
-                hsfl[i].copy_(o["sf_linear"], non_blocking=True)
-                hsfs[i].copy_(o["sf_swizzled"], non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record(stream)
+                done.append(ev)
+            with torch.cuda.stream(down):
+                for i in range(len(xs)):
+                    down.wait_event(done[i])
+                    o = eouts[i]
+                    hcodes[i].copy_(o["codes"], non_blocking=True)
+                    hsfl[i].copy_(o["sf_linear"], non_blocking=True)
+                    hsfs[i].copy_(o["sf_swizzled"], non_blocking=True)
+            stream.wait_stream(down)
 
         e_reps = max(3, min(20, args.steps))
         t_e2e = time_leg(e2e_step, e_reps)
         h2d = sum(x.numel() * x.element_size() for x in xs)
         d2h = sum(o["codes"].numel() + o["sf_linear"].numel() + o["sf_swizzled"].numel() for o in outs)
+
+        def h2d_only():
+            for i in range(len(xs)):
+                dx[i].copy_(hx[i], non_blocking=True)
+
+        t_h2d = time_leg(h2d_only, e_reps)
         e2e = {"value": round(world * total / (t_e2e * 1e-3) / 1e9, 3), "unit": "Gelem/s",
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(t_e2e, 4)}
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(t_e2e, 4),
+               "h2d_gb_s_alone": round(h2d / (t_h2d * 1e-3) / 1e9, 1),
+               "streams": "H2D, compute and D2H on three streams, event-ordered per tensor"}
 
     # ---- CPU baseline: the oracle on a bounded sample, rank 0 at N = 1 only
     cpu = None
