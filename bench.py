@@ -195,15 +195,26 @@ def run_gpu(args, rank, world):
         B.scalesweep_quantize(xs[i], 16, S[i:i + 1], B.NVFP4_OBJ_WMSE, ws[i], 0, *win, o["codes"], o["sf_linear"],
                               o["sf_swizzled"], None, stream=stream)
 
+    aux = torch.cuda.Stream()
+    wsps = [torch.empty_like(wsp) for _ in xs]
+    amax_done = [torch.cuda.Event() for _ in xs]
+
     def step(events=None):
-        for i, x in enumerate(xs):
-            B.nvfp4_global_scale(x, D, S[i:i + 1], st, wsp, stream=stream)
+        # The global scales run on a side stream: amax(i+1) (HBM-bound) overlaps
+        # sweep(i) (ALU-bound); sweep(i) waits only for amax(i).
+        aux.wait_stream(stream)
+        with torch.cuda.stream(aux):
+            for i, x in enumerate(xs):
+                B.nvfp4_global_scale(x, D, S[i:i + 1], st, wsps[i], stream=aux)
+                amax_done[i].record(aux)
         for i in range(len(xs)):
+            stream.wait_event(amax_done[i])
             if events is not None:
                 events[i][0].record(stream)
             sweep(i)
             if events is not None:
                 events[i][1].record(stream)
+        stream.wait_stream(aux)
 
     launches_per_step = 3 * len(xs)   # amax partial + final + sweep per tensor (shapes need no pad kernel)
 

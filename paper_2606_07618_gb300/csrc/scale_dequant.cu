@@ -115,16 +115,19 @@ cudaError_t launch_global_scale(const void* x, int dtype, int64_t n, float fp8_d
                                 int* status_dev, void* ws, int sms, cudaStream_t s) {
     float* part_max = static_cast<float*>(ws);
     int* part_bad = reinterpret_cast<int*>(part_max + kAmaxParts);
+    // 128-thread CTAs (~4K registers each) so the reduction can share SMs with
+    // an ALU-bound sweep running on another stream.
+    constexpr int kThreads = 128;
     const int per = dtype == 0 ? 8 : 4;
     const int64_t nvec = n / per;
-    int64_t grid = (nvec + 255) / 256;
-    if (grid > (int64_t)sms * 4) grid = (int64_t)sms * 4;
+    int64_t grid = (nvec + kThreads * 4 - 1) / (kThreads * 4);
+    if (grid > (int64_t)sms * 6) grid = (int64_t)sms * 6;
     if (grid > kAmaxParts) grid = kAmaxParts;
     if (grid < 1) grid = 1;
     if (dtype == 0)
-        amax_partial_kernel<0><<<(int)grid, 256, 0, s>>>(x, n, part_max, part_bad);
+        amax_partial_kernel<0><<<(int)grid, kThreads, 0, s>>>(x, n, part_max, part_bad);
     else
-        amax_partial_kernel<1><<<(int)grid, 256, 0, s>>>(x, n, part_max, part_bad);
+        amax_partial_kernel<1><<<(int)grid, kThreads, 0, s>>>(x, n, part_max, part_bad);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     amax_final_kernel<<<1, 256, 0, s>>>(part_max, part_bad, (int)grid, fp8_div, S_out, status_dev);
