@@ -513,6 +513,62 @@ def run_kernel_case(args):
                       "ms": round(ms, 4), "gelem_s": round(n / ms / 1e6, 2)}), flush=True)
 
 
+def run_table7(args):
+    """Latency of the NVFP4 quantisation operator at hidden 8192 for the batch
+    sizes of the paper's latency table (Appendix E, Table 7), on this GPU:
+    per-call global scale + ScaleSweep (MSE and WMSE) or AbsMax, both scale
+    layouts, timed with CUDA events (context for the paper's RTX PRO 6000
+    figures, not a like-for-like comparison)."""
+    from paper_2606_07618_gb300 import binding as B
+    from paper_2606_07618_gb300 import workloads as W
+    dev = "cuda"
+    win = (B.NVFP4_WINDOW_DEFAULT, B.NVFP4_WINDOW_DEFAULT)
+    rows = []
+    for b in (128, 256, 512, 1024, 2048, 4096, 8192, 16384, 32768):
+        t = W.workload(f"table7-{b}").tensors[0]
+        x = W.draw(t).to(dev)
+        w = torch.exp(torch.randn(t.cols, generator=torch.Generator().manual_seed(b))).to(dev)
+        S = torch.empty(1, device=dev)
+        ws = torch.empty(B.nvfp4_global_scale_workspace(x.numel()), dtype=torch.uint8, device=dev)
+        o = B.empty_outputs(b, t.cols, 16, device=dev, linear=True, swizzled=True)
+
+        B.nvfp4_global_scale(x, 256.0, S, None, ws)     # static scale: computed once, as in the paper
+
+        def op(kind):
+            def f():
+                if kind.endswith("_dyn"):
+                    B.nvfp4_global_scale(x, 256.0, S, None, ws)
+                    kind_ = kind[:-4]
+                else:
+                    kind_ = kind
+                if kind_ == "absmax":
+                    B.absmax_quantize(x, 16, S, o["codes"], o["sf_linear"], o["sf_swizzled"])
+                else:
+                    obj = B.NVFP4_OBJ_WMSE if kind_ == "wmse" else B.NVFP4_OBJ_MSE
+                    B.scalesweep_quantize(x, 16, S, obj, w if kind_ == "wmse" else None, 0, *win, o["codes"],
+                                          o["sf_linear"], o["sf_swizzled"])
+            return f
+
+        res = {"batch": b}
+        for kind in ("absmax", "mse", "wmse", "absmax_dyn", "mse_dyn", "wmse_dyn"):
+            f = op(kind)
+            for _ in range(5):
+                f()
+            torch.cuda.synchronize()
+            a, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            reps = 50
+            a.record()
+            for _ in range(reps):
+                f()
+            e.record()
+            torch.cuda.synchronize()
+            res[kind + "_ms"] = round(a.elapsed_time(e) / reps, 4)
+        res["mse_rel"] = round(res["mse_ms"] / res["absmax_ms"], 3)
+        res["wmse_rel"] = round(res["wmse_ms"] / res["absmax_ms"], 3)
+        rows.append(res)
+        print(json.dumps(res), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -529,7 +585,11 @@ def main():
     ap.add_argument("--cols", type=int, default=8192)
     ap.add_argument("--block", type=int, default=16)
     ap.add_argument("--reps", type=int, default=5)
+    ap.add_argument("--table7", action="store_true")
     args = ap.parse_args()
+    if args.table7:
+        run_table7(args)
+        return
     if args.kernel_case:
         run_kernel_case(args)
         return

@@ -9,8 +9,9 @@ float32 for the rounding decisions the kernels also take in float32); this
 module builds it with gcc and wraps it for numpy arrays.  ``bounds.py`` holds
 the exact rational re-derivations of the paper's bit-pattern bounds.
 
-Parity unpinned: ``swizzle_scales`` (the 128x4 scale-factor layout is defined by
-NVIDIA's block-scaling documentation, not by the paper).
+``swizzle_scales`` (the 128x4 scale-factor layout, defined by NVIDIA's block-scaling
+layout rather than by the paper) is pinned on the GPU against cuBLASLt's NVFP4
+block-scaled GEMM.
 """
 from __future__ import annotations
 

@@ -35,9 +35,9 @@
  * force and against torch's float8_e4m3fn, Lemma-4.2/4.3 tables and the convex
  * certificates recomputed, bounded = exhaustive sweep, ScaleSweep <= AbsMax and
  * <= 4/6, Appendix-C optimum <= every FP8 result, closed-form blocks.
- * Parity unpinned: the 128x4 swizzled scale layout (oracle_swizzle_scales) is an
- * index permutation taken from NVIDIA's public block-scaling layout description;
- * the paper does not define it and no independent reference is available on CPU.
+ * The 128x4 swizzled scale layout (oracle_swizzle_scales) is not defined by the
+ * paper; it follows NVIDIA's block-scaling layout and is pinned on the GPU
+ * against cuBLASLt's NVFP4 block-scaled GEMM (tests/test_gpu_swizzle_pin.py).
  */
 #include <math.h>
 #include <stdint.h>

@@ -126,6 +126,10 @@ __device__ __forceinline__ uint32_t fast_div(uint32_t n, const FastDiv& d) {
 #ifndef NVFP4_QMINB
 #define NVFP4_QMINB 1
 #endif
+#ifndef NVFP4_CAND_UNROLL
+#define NVFP4_CAND_UNROLL 16
+#endif
+constexpr int kCandUnroll = NVFP4_CAND_UNROLL;
 
 // FIX = 1: default window (fixed length, unrolled, poison-padded table).
 template <int DT, int METHOD, int OBJ, int BLOCK, int FIX>
@@ -214,7 +218,7 @@ __global__ void __launch_bounds__(256, NVFP4_QMINB) quantize_kernel(QuantParams 
             if (FIX) {
                 const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
                 int bk = 0;
-#pragma unroll
+#pragma unroll kCandUnroll
                 for (int k = 0; k < FIX_K; k++) {
                     const Cand cd = tb[k];
                     const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));

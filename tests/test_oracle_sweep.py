@@ -338,9 +338,10 @@ def test_dequantize_matches_format_tables(oracle_mod):
 
 @pytest.mark.parametrize("rows,kb", [(1, 1), (130, 5), (128, 4), (256, 8), (300, 13)])
 def test_swizzle_layout_structure(oracle_mod, rows, kb):
-    """Parity unpinned (layout from NVIDIA's block-scaling description); these
-    are structural checks only: a bijection into the padded buffer, zero pads,
-    512-byte 128x4 atoms, rows r, r+32, r+64, r+96 sharing one 16-byte line."""
+    """Structural checks of the swizzled layout on CPU (the layout itself is
+    pinned against cuBLASLt in test_gpu_swizzle_pin.py): a bijection into the
+    padded buffer, zero pads, 512-byte 128x4 atoms, rows r, r+32, r+64, r+96
+    sharing one 16-byte line."""
     nbytes = oracle_mod.swizzle_bytes(rows, kb)
     assert nbytes == -(-rows // 128) * 128 * (-(-kb // 4)) * 4
     offs = {oracle_mod.swizzle_offset(r, k, kb) for r in range(rows) for k in range(kb)}
