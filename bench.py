@@ -485,6 +485,7 @@ def run_kernel_case(args):
     o = B.empty_outputs(args.rows, args.cols, args.block, device=dev, linear=True, swizzled=args.block == 16)
     win = (B.NVFP4_WINDOW_DEFAULT, B.NVFP4_WINDOW_DEFAULT)
     dq = torch.empty(args.rows, args.cols, dtype=torch.bfloat16, device=dev)
+    dws = torch.empty(B.nvfp4_dynamic_workspace(), dtype=torch.uint8, device=dev)
     fns = {
         "sweep_wmse": lambda: B.scalesweep_quantize(x, args.block, S, 1, w, 0, *win, o["codes"], o["sf_linear"],
                                                     o["sf_swizzled"]),
@@ -495,6 +496,13 @@ def run_kernel_case(args):
                                                      o["sf_swizzled"]),
         "dequant": lambda: B.nvfp4_dequantize(o["codes"], o["sf_linear"], 1, S, args.rows, args.cols, args.block, dq),
         "amax": lambda: B.nvfp4_global_scale(x, 256.0, S, None, ws),
+        "mse_two_launch": lambda: (B.nvfp4_global_scale(x, 256.0, S, None, ws),
+                                   B.scalesweep_quantize(x, args.block, S, 0, None, 0, *win, o["codes"],
+                                                         o["sf_linear"], o["sf_swizzled"])),
+        "mse_fused": lambda: B.scalesweep_quantize_dynamic(x, args.block, 256.0, 0, None, 0, *win, S, None, dws,
+                                                           o["codes"], o["sf_linear"], o["sf_swizzled"]),
+        "wmse_fused": lambda: B.scalesweep_quantize_dynamic(x, args.block, 256.0, 1, w, 0, *win, S, None, dws,
+                                                            o["codes"], o["sf_linear"], o["sf_swizzled"]),
     }
     fn = fns[args.kernel_case]
     fns["sweep_mse"]()
@@ -533,9 +541,20 @@ def run_table7(args):
         o = B.empty_outputs(b, t.cols, 16, device=dev, linear=True, swizzled=True)
 
         B.nvfp4_global_scale(x, 256.0, S, None, ws)     # static scale: computed once, as in the paper
+        dws = torch.empty(B.nvfp4_dynamic_workspace(), dtype=torch.uint8, device=dev)
+        S2 = torch.empty(1, device=dev)
 
         def op(kind):
             def f():
+                if kind.endswith("_fused"):
+                    if kind.startswith("absmax"):
+                        B.absmax_quantize_dynamic(x, 16, 256.0, S2, None, dws, o["codes"], o["sf_linear"],
+                                                  o["sf_swizzled"])
+                    else:
+                        obj = B.NVFP4_OBJ_WMSE if kind.startswith("wmse") else B.NVFP4_OBJ_MSE
+                        B.scalesweep_quantize_dynamic(x, 16, 256.0, obj, w if obj else None, 0, *win, S2, None,
+                                                      dws, o["codes"], o["sf_linear"], o["sf_swizzled"])
+                    return
                 if kind.endswith("_dyn"):
                     B.nvfp4_global_scale(x, 256.0, S, None, ws)
                     kind_ = kind[:-4]
@@ -550,7 +569,8 @@ def run_table7(args):
             return f
 
         res = {"batch": b}
-        for kind in ("absmax", "mse", "wmse", "absmax_dyn", "mse_dyn", "wmse_dyn"):
+        for kind in ("absmax", "mse", "wmse", "absmax_dyn", "mse_dyn", "wmse_dyn", "absmax_fused", "mse_fused",
+                     "wmse_fused"):
             f = op(kind)
             for _ in range(5):
                 f()
@@ -580,7 +600,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-rows", type=int, default=64)
     ap.add_argument("--kernel-case", default=None,
-                    choices=["sweep_wmse", "sweep_mse", "absmax", "four_six", "dequant", "amax"])
+                    choices=["sweep_wmse", "sweep_mse", "absmax", "four_six", "dequant", "amax", "mse_two_launch",
+                             "mse_fused", "wmse_fused"])
     ap.add_argument("--rows", type=int, default=16384)
     ap.add_argument("--cols", type=int, default=8192)
     ap.add_argument("--block", type=int, default=16)

@@ -138,6 +138,42 @@ nvfp4_status scalesweep_quantize(const void* x, nvfp4_dtype dt, int64_t rows, in
                                  uint8_t* sf_swizzled, float* block_loss, void* stream);
 
 /*
+ * Bytes of device workspace the *_quantize_dynamic entry points need.
+ */
+size_t nvfp4_dynamic_workspace(void);
+
+/*
+ * ScaleSweep quantisation with a per-call (dynamic) global scale computed in
+ * the same launch: S = fl32(amax / fl32(6*fp8_div)) (Sec. 4.2.1) over the whole
+ * tensor, then the sweep of scalesweep_quantize with that S.  This fuses the
+ * reduction into the sweep for dynamic activation quantisation (the paper's
+ * kernels leave fusion as future work, Sec. 5.2).  One cooperative launch (all
+ * CTAs resident) with a grid barrier in between, preceded by a 4-byte
+ * cudaMemsetAsync of the barrier counter in the workspace.
+ *   S_out       device float written with S (also returned implicitly by the codes).
+ *   status_dev  optional device int: bit 0 OR-ed in for NaN/inf input, bit 1 if the
+ *               grid barrier timed out (about a second; the outputs are then not
+ *               written -- a resident grid makes this unreachable in practice).
+ *   workspace   nvfp4_dynamic_workspace() bytes, 16-byte aligned, no initialisation.
+ * Other arguments as scalesweep_quantize.  rows*cols == 0 launches nothing.
+ * Concurrent calls must use distinct workspaces.
+ */
+nvfp4_status scalesweep_quantize_dynamic(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                                         float fp8_div, nvfp4_objective obj, const float* w, int64_t w_row_stride,
+                                         int win_lo, int win_hi, float* S_out, int* status_dev, void* workspace,
+                                         size_t ws_bytes, uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled,
+                                         float* block_loss, void* stream);
+
+/*
+ * AbsMax quantisation with the global scale computed in the same launch, as
+ * scalesweep_quantize_dynamic (baseline for the fused dynamic path).
+ */
+nvfp4_status absmax_quantize_dynamic(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                                     float fp8_div, float* S_out, int* status_dev, void* workspace, size_t ws_bytes,
+                                     uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled, float* block_loss,
+                                     void* stream);
+
+/*
  * AbsMax quantisation (Sec. 3.2): s = max(1, RN_E4M3(s_base)) as a code (a block
  * whose RN scale would be 0 gets the smallest positive scale), q = RNE_E2M1.
  * Arguments as scalesweep_quantize; block_loss is the MSE loss of the chosen

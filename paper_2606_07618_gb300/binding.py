@@ -55,8 +55,12 @@ def lib() -> ctypes.CDLL:
         L.absmax_quantize.argtypes = [p, i, i64, i64, i, p, p, p, p, p, p]
         L.four_over_six_quantize.argtypes = [p, i, i64, i64, i, p, i, p, i64, p, p, p, p, p]
         L.nvfp4_dequantize.argtypes = [p, p, i, p, i64, i64, i, p, i, p]
+        L.nvfp4_dynamic_workspace.argtypes, L.nvfp4_dynamic_workspace.restype = [], sz
+        L.scalesweep_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, i, p, i64, i, i, p, p, p, sz, p, p, p, p, p]
+        L.absmax_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, p, p, p, sz, p, p, p, p, p]
         for fn in ("nvfp4_global_scale", "nvfp4_global_scale_noalloc", "scalesweep_quantize", "absmax_quantize",
-                   "four_over_six_quantize", "nvfp4_dequantize"):
+                   "four_over_six_quantize", "nvfp4_dequantize", "scalesweep_quantize_dynamic",
+                   "absmax_quantize_dynamic"):
             getattr(L, fn).restype = i
         _lib = L
     return _lib
@@ -137,6 +141,32 @@ def four_over_six_quantize(x, block: int, S, objective: int, w, w_row_stride: in
                                       int(w_row_stride), _ptr(codes), _ptr(sf_linear), _ptr(sf_swizzled),
                                       _ptr(block_loss), _stream(stream))
     _check("four_over_six_quantize", rc)
+
+
+def nvfp4_dynamic_workspace() -> int:
+    return int(lib().nvfp4_dynamic_workspace())
+
+
+def scalesweep_quantize_dynamic(x, block: int, fp8_div: float, objective: int, w, w_row_stride: int, win_lo: int,
+                                win_hi: int, S_out, status, workspace, codes, sf_linear=None, sf_swizzled=None,
+                                block_loss=None, stream=None):
+    rows, cols = x.shape
+    ws_bytes = workspace.numel() * workspace.element_size()
+    rc = lib().scalesweep_quantize_dynamic(_ptr(x), _dtype(x), rows, cols, int(block), float(fp8_div), int(objective),
+                                           _ptr(w), int(w_row_stride), int(win_lo), int(win_hi), _ptr(S_out),
+                                           _ptr(status), _ptr(workspace), ws_bytes, _ptr(codes), _ptr(sf_linear),
+                                           _ptr(sf_swizzled), _ptr(block_loss), _stream(stream))
+    _check("scalesweep_quantize_dynamic", rc)
+
+
+def absmax_quantize_dynamic(x, block: int, fp8_div: float, S_out, status, workspace, codes, sf_linear=None,
+                            sf_swizzled=None, block_loss=None, stream=None):
+    rows, cols = x.shape
+    ws_bytes = workspace.numel() * workspace.element_size()
+    rc = lib().absmax_quantize_dynamic(_ptr(x), _dtype(x), rows, cols, int(block), float(fp8_div), _ptr(S_out),
+                                       _ptr(status), _ptr(workspace), ws_bytes, _ptr(codes), _ptr(sf_linear),
+                                       _ptr(sf_swizzled), _ptr(block_loss), _stream(stream))
+    _check("absmax_quantize_dynamic", rc)
 
 
 def nvfp4_dequantize(codes, sf, layout: int, S, rows: int, cols: int, block: int, out, stream=None):

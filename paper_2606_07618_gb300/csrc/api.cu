@@ -77,10 +77,19 @@ nvfp4_status check_shape(int64_t rows, int64_t cols, int block, Shape* sh) {
     return NVFP4_OK;
 }
 
+// Extra arguments of the dynamic-scale variants (global scale computed in the launch).
+struct DynArgs {
+    float fp8_div;
+    float* S_out;
+    int* status_dev;
+    void* workspace;
+    size_t ws_bytes;
+};
+
 nvfp4_status quantize_common(int method, const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
                              const float* S, nvfp4_objective obj, const float* w, int64_t w_row_stride,
                              int win_lo, int win_hi, uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled,
-                             float* block_loss, void* stream) {
+                             float* block_loss, void* stream, const DynArgs* dyn = nullptr) {
     if (dt != NVFP4_IN_BF16 && dt != NVFP4_IN_F32) return NVFP4_ERR_INVALID_ARG;
     if (obj != NVFP4_OBJ_MSE && obj != NVFP4_OBJ_WMSE) return NVFP4_ERR_INVALID_ARG;
     Shape sh;
@@ -94,6 +103,13 @@ nvfp4_status quantize_common(int method, const void* x, nvfp4_dtype dt, int64_t 
         } else if (win_lo < -126 || win_hi > 126 || win_lo > win_hi) {
             return NVFP4_ERR_INVALID_ARG;
         }
+    }
+    if (dyn) {
+        if (!(dyn->fp8_div > 0.0f) || dyn->fp8_div > 1e30f) return NVFP4_ERR_INVALID_ARG;
+        if (!dyn->S_out || !dyn->workspace || dyn->ws_bytes < kDynWorkspace) return NVFP4_ERR_INVALID_ARG;
+        if (!aligned(dyn->workspace, 16) || !aligned(dyn->S_out, 4) || (dyn->status_dev && !aligned(dyn->status_dev, 4)))
+            return NVFP4_ERR_ALIGNMENT;
+        S = dyn->S_out;
     }
     if (sh.n == 0) return NVFP4_OK;
     if (!x || !S || !codes || (!sf_linear && !sf_swizzled)) return NVFP4_ERR_INVALID_ARG;
@@ -117,18 +133,21 @@ nvfp4_status quantize_common(int method, const void* x, nvfp4_dtype dt, int64_t 
         }
     }
     const int64_t cbytes = sh.n / 2, lbytes = sh.nblocks, sbytes = sh.sw_bytes, fbytes = sh.nblocks * 4;
-    const void* outs[4] = {codes, sf_linear, sf_swizzled, block_loss};
-    const int64_t olen[4] = {cbytes, lbytes, sbytes, fbytes};
-    for (int i = 0; i < 4; i++) {
+    const void* outs[7] = {codes, sf_linear, sf_swizzled, block_loss, dyn ? dyn->workspace : nullptr,
+                           dyn ? (const void*)dyn->status_dev : nullptr, dyn ? (const void*)dyn->S_out : nullptr};
+    const int64_t olen[7] = {cbytes, lbytes, sbytes, fbytes, dyn ? (int64_t)dyn->ws_bytes : 0, 4, 4};
+    for (int i = 0; i < 7; i++) {
         if (!outs[i]) continue;
-        if (overlap(outs[i], olen[i], x, xbytes) || overlap(outs[i], olen[i], S, 4)) return NVFP4_ERR_INVALID_ARG;
+        if (overlap(outs[i], olen[i], x, xbytes)) return NVFP4_ERR_INVALID_ARG;
+        if (!dyn && overlap(outs[i], olen[i], S, 4)) return NVFP4_ERR_INVALID_ARG;
         if (obj == NVFP4_OBJ_WMSE && overlap(outs[i], olen[i], w, wbytes)) return NVFP4_ERR_INVALID_ARG;
-        for (int j = i + 1; j < 4; j++)
+        for (int j = i + 1; j < 7; j++)
             if (overlap(outs[i], olen[i], outs[j], olen[j])) return NVFP4_ERR_INVALID_ARG;
     }
     if (!device_accessible(x) || !device_accessible(S) || !device_accessible(codes) ||
         !device_accessible(sf_linear) || !device_accessible(sf_swizzled) || !device_accessible(block_loss) ||
-        (obj == NVFP4_OBJ_WMSE && !device_accessible(w)))
+        (obj == NVFP4_OBJ_WMSE && !device_accessible(w)) ||
+        (dyn && (!device_accessible(dyn->workspace) || !device_accessible(dyn->status_dev))))
         return NVFP4_ERR_INVALID_ARG;
     const int sms = sm_count();
     if (sms <= 0) return NVFP4_ERR_CUDA;
@@ -150,8 +169,25 @@ nvfp4_status quantize_common(int method, const void* x, nvfp4_dtype dt, int64_t 
     p.sf_linear = sf_linear;
     p.sf_swizzled = sf_swizzled;
     p.block_loss = block_loss;
-    cudaError_t e = launch_quantize(p, dt == NVFP4_IN_BF16 ? 0 : 1, method, obj == NVFP4_OBJ_WMSE ? 1 : 0, block,
-                                    sms, static_cast<cudaStream_t>(stream));
+    p.fp8_div = 0.0f;
+    p.S_out = nullptr;
+    p.status_dev = nullptr;
+    p.part_max = nullptr;
+    p.part_bad = nullptr;
+    p.barrier = nullptr;
+    const int dti = dt == NVFP4_IN_BF16 ? 0 : 1, obji = obj == NVFP4_OBJ_WMSE ? 1 : 0;
+    cudaError_t e;
+    if (dyn) {
+        p.fp8_div = dyn->fp8_div;
+        p.S_out = dyn->S_out;
+        p.status_dev = dyn->status_dev;
+        p.part_max = static_cast<float*>(dyn->workspace);
+        p.part_bad = reinterpret_cast<int*>(p.part_max + kAmaxParts);
+        p.barrier = reinterpret_cast<unsigned*>(p.part_bad + kAmaxParts);
+        e = launch_quantize_dynamic(p, dti, method, obji, block, sms, static_cast<cudaStream_t>(stream));
+    } else {
+        e = launch_quantize(p, dti, method, obji, block, sms, static_cast<cudaStream_t>(stream));
+    }
     return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
 }
 
@@ -207,6 +243,27 @@ nvfp4_status scalesweep_quantize(const void* x, nvfp4_dtype dt, int64_t rows, in
                                  uint8_t* sf_swizzled, float* block_loss, void* stream) {
     return quantize_common(0, x, dt, rows, cols, block, S, obj, w, w_row_stride, win_lo, win_hi, codes, sf_linear,
                            sf_swizzled, block_loss, stream);
+}
+
+size_t nvfp4_dynamic_workspace(void) { return kDynWorkspace; }
+
+nvfp4_status scalesweep_quantize_dynamic(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                                         float fp8_div, nvfp4_objective obj, const float* w, int64_t w_row_stride,
+                                         int win_lo, int win_hi, float* S_out, int* status_dev, void* workspace,
+                                         size_t ws_bytes, uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled,
+                                         float* block_loss, void* stream) {
+    const DynArgs d{fp8_div, S_out, status_dev, workspace, ws_bytes};
+    return quantize_common(0, x, dt, rows, cols, block, nullptr, obj, w, w_row_stride, win_lo, win_hi, codes,
+                           sf_linear, sf_swizzled, block_loss, stream, &d);
+}
+
+nvfp4_status absmax_quantize_dynamic(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                                     float fp8_div, float* S_out, int* status_dev, void* workspace, size_t ws_bytes,
+                                     uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled, float* block_loss,
+                                     void* stream) {
+    const DynArgs d{fp8_div, S_out, status_dev, workspace, ws_bytes};
+    return quantize_common(1, x, dt, rows, cols, block, nullptr, NVFP4_OBJ_MSE, nullptr, 0, 0, 0, codes, sf_linear,
+                           sf_swizzled, block_loss, stream, &d);
 }
 
 nvfp4_status absmax_quantize(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,

@@ -26,17 +26,34 @@ struct QuantParams {
     uint8_t* sf_linear;
     uint8_t* sf_swizzled;
     float* block_loss;
+    // dynamic (per-call) global scale, computed inside the sweep launch
+    float fp8_div;
+    float* S_out;
+    int* status_dev;
+    float* part_max;
+    int* part_bad;
+    unsigned* barrier;
 };
 
 // dtype 0 bf16 / 1 f32; method 0 ScaleSweep / 1 AbsMax / 2 four-over-six;
 // obj 0 MSE / 1 WMSE; block 16/32/64; sms = multiprocessor count.
 cudaError_t launch_quantize(const QuantParams& p, int dtype, int method, int obj, int block, int sms,
                             cudaStream_t s);
+// Same with the global scale computed in the launch (method 0 or 1; p.S unused,
+// p.S_out/part_max/part_bad/barrier in the caller's workspace).
+cudaError_t launch_quantize_dynamic(const QuantParams& p, int dtype, int method, int obj, int block, int sms,
+                                    cudaStream_t s);
+// Zero the pads of a swizzled scale buffer when rows % 128 or kb % 4 != 0.
+cudaError_t launch_swizzle_pad(const QuantParams& p, int sms, cudaStream_t s);
+// Fill the derived fields of p (window mode, row/column need, fast divider).
+void prepare_quant_params(QuantParams& p, int method, int obj, int block, bool* fix);
 
 // Global-scale reduction: partial maxima into ws, then S and the status word.
 cudaError_t launch_global_scale(const void* x, int dtype, int64_t n, float fp8_div, float* S_out,
                                 int* status_dev, void* ws, int sms, cudaStream_t s);
 constexpr int kAmaxParts = 1024;   // partial slots in the workspace
+// Dynamic-scale workspace: partial maxima, partial flags, barrier counter.
+constexpr size_t kDynWorkspace = (size_t)kAmaxParts * 8 + 256;
 
 // Same two kernels with caller-chosen partial slots and grid (grid <= slots).
 cudaError_t launch_global_scale_parts(const void* x, int dtype, int64_t n, float fp8_div, float* S_out,

@@ -1,0 +1,449 @@
+// NVFP4 block-scale selection kernels: ScaleSweep (Sec. 4.2.2 of the paper),
+// AbsMax (Sec. 3.2) and 4/6 (Sec. 2), sharing one register-resident skeleton.
+//
+// Mapping: one thread owns one 16-element segment (32 or 64 bytes of input) and
+// keeps it in registers; a scale block of 16/32/64 elements is 1/2/4
+// consecutive lanes of a warp, which combine block max and per-candidate losses
+// with xor-shuffles (commutative pairwise sums, so every lane of a block holds
+// bit-identical losses and takes the same decision).  The grid-stride loop
+// walks whole warps so every shuffle runs with all 32 lanes converged, and the
+// next segment's input is loaded before the current one is swept.
+//
+// ScaleSweep per block: y = fl(x*E), m = max|y|, s_base = fl(m/6),
+// I0 = floor_E4M3(s_base); for codes c in [I0+lo, I0+hi] clamped to 1..126:
+// L_c = sum_i w_i (y_i - q_i v_c)^2 with q_i = RNE_E2M1(fl(y_i * fl(1/v_c)));
+// keep the first (lowest-code) minimum.  The per-candidate work on an element
+// pair is mul.f32x2 -> cvt e2m1x2 -> cvt f16x2 (exact decode) -> two mixed
+// fma.f32.f16 (exact product q*(-v), one rounding) -> fma.f32x2 accumulate.
+//
+// Candidate table: entry code+128 holds {fl(1/v_c), f16 bits of -v_c} for codes
+// 1..126 and a poison entry {+inf, -inf} elsewhere.  A poison candidate's loss
+// is inf or NaN, so it never wins the strict "<" -- this lets the default
+// windows run a fixed, fully unrolled loop over [I0+lo, I0+hi] with no clamping
+// (those windows always contain a real code).  Custom windows clamp instead.
+#pragma once
+#include "nvfp4_device.cuh"
+#include "nvfp4_kernels.h"
+
+namespace nvfp4 {
+
+struct Cand {
+    float r;        // fl(1/v_c)
+    uint32_t nv;    // f16 bits of -v_c in the low half
+};
+constexpr int kTabOff = 128;
+constexpr int kTabN = 384;
+
+__device__ __forceinline__ void build_table(Cand* t) {
+    for (int i = threadIdx.x; i < kTabN; i += blockDim.x) {
+        const int c = i - kTabOff;
+        Cand e;
+        if (c >= 1 && c <= 126) {
+            const uint16_t h = e4m3_to_f16bits((uint32_t)c);
+            e.r = __frcp_rn(f16bits_to_f32(h));
+            e.nv = (uint32_t)(h ^ 0x8000u);
+        } else {
+            e.r = __int_as_float(0x7f800000);
+            e.nv = 0xFC00u;
+        }
+        t[i] = e;
+    }
+}
+
+struct Raw {
+    uint4 a, b, c, d;
+};
+
+template <int DT>
+__device__ __forceinline__ void load_raw(const void* x, int64_t g, Raw& r) {
+    if (DT == 0) {
+        const uint4* p = reinterpret_cast<const uint4*>(static_cast<const char*>(x) + g * 32);
+        r.a = ld_stream16(p);
+        r.b = ld_stream16(p + 1);
+    } else {
+        const uint4* p = reinterpret_cast<const uint4*>(static_cast<const char*>(x) + g * 64);
+        r.a = ld_stream16(p);
+        r.b = ld_stream16(p + 1);
+        r.c = ld_stream16(p + 2);
+        r.d = ld_stream16(p + 3);
+    }
+}
+
+template <int DT>
+__device__ __forceinline__ void raw_to_float(const Raw& r, float (&xv)[16]) {
+    if (DT == 0) {
+        const uint32_t u[8] = {r.a.x, r.a.y, r.a.z, r.a.w, r.b.x, r.b.y, r.b.z, r.b.w};
+#pragma unroll
+        for (int j = 0; j < 8; j++) {
+            xv[2 * j] = bf16lo(u[j]);
+            xv[2 * j + 1] = bf16hi(u[j]);
+        }
+    } else {
+        const uint32_t u[16] = {r.a.x, r.a.y, r.a.z, r.a.w, r.b.x, r.b.y, r.b.z, r.b.w,
+                                r.c.x, r.c.y, r.c.z, r.c.w, r.d.x, r.d.y, r.d.z, r.d.w};
+#pragma unroll
+        for (int j = 0; j < 16; j++) xv[j] = __uint_as_float(u[j]);
+    }
+}
+
+// Loss of one candidate on this thread's 16 elements.
+template <int OBJ>
+__device__ __forceinline__ float seg_loss(const u64 (&y2)[8], const u64 (&w2)[8], float r, uint16_t nv) {
+    const u64 r2 = pack2(r, r);
+    u64 acc = 0ull;
+#pragma unroll
+    for (int j = 0; j < 8; j++) {
+        const u64 e2 = cand_err2(y2[j], r2, nv);
+        if (OBJ == 1) {
+            acc = fma2(mul2(w2[j], e2), e2, acc);
+        } else {
+            acc = fma2(e2, e2, acc);
+        }
+    }
+    float a, b;
+    unpack2(acc, a, b);
+    return __fadd_rn(a, b);
+}
+
+template <int SEGS>
+__device__ __forceinline__ float group_sum(float v) {
+    if (SEGS >= 2) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, 1));
+    if (SEGS >= 4) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, 2));
+    return v;
+}
+template <int SEGS>
+__device__ __forceinline__ float group_max(float v) {
+    if (SEGS >= 2) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 1));
+    if (SEGS >= 4) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 2));
+    return v;
+}
+
+// n / d for 32-bit n by multiply-high and shifts (Granlund-Montgomery).
+__device__ __forceinline__ uint32_t fast_div(uint32_t n, const FastDiv& d) {
+    const uint32_t t = __umulhi(n, d.mul);
+    return (t + ((n - t) >> d.s1)) >> d.s2;
+}
+
+#ifndef NVFP4_QMINB
+#define NVFP4_QMINB 1
+#endif
+#ifndef NVFP4_CAND_UNROLL
+#define NVFP4_CAND_UNROLL 16
+#endif
+constexpr int kCandUnroll = NVFP4_CAND_UNROLL;
+
+// Dynamic (per-call) global scale inside the sweep launch: every CTA folds the
+// max |x| of its grid-stride share into one partial, all CTAs meet at a grid
+// barrier (cooperative launch, so all are resident; the counter is zeroed by
+// the host before the launch), then each CTA folds all partials into the same
+// S = fl(amax / fl(6 D)).  The barrier wait is bounded: on timeout the kernel
+// sets bit 1 of the status word and returns without writing outputs.
+constexpr unsigned kBarrierSpinLimit = 1u << 24;
+
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+template <int DT>
+__device__ __forceinline__ bool dynamic_scale(const QuantParams& p, float& S_out) {
+    __shared__ uint32_t sm[32];
+    __shared__ int sb[32];
+    __shared__ int s_timeout;
+    constexpr int PER = DT == 0 ? 8 : 4;
+    const int64_t nvec = (p.nseg * 16) / PER;
+    const uint4* xv = static_cast<const uint4*>(p.x);
+    float m = 0.0f;
+    int bad = 0;
+    auto fold = [&](const uint4& u) {
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            if (DT == 0) {
+                const float a = bf16lo(w[j]), b = bf16hi(w[j]);
+                bad |= (!isfinite(a)) | (!isfinite(b));
+                m = fmaxf(m, fmaxf(fabsf(a), fabsf(b)));
+            } else {
+                const float a = __uint_as_float(w[j]);
+                bad |= !isfinite(a);
+                m = fmaxf(m, fabsf(a));
+            }
+        }
+    };
+    const int64_t gstride = (int64_t)gridDim.x * blockDim.x;
+    int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    for (; i + 7 * gstride < nvec; i += 8 * gstride) {      // eight 16-byte loads in flight per thread
+        uint4 u[8];
+#pragma unroll
+        for (int j = 0; j < 8; j++) u[j] = ld_stream16(xv + i + j * gstride);
+#pragma unroll
+        for (int j = 0; j < 8; j++) fold(u[j]);
+    }
+    for (; i < nvec; i += gstride) fold(ld_stream16(xv + i));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+    uint32_t mb = __reduce_max_sync(0xffffffffu, __float_as_uint(m));
+    int wb = __reduce_or_sync(0xffffffffu, (unsigned)bad);
+    if (lane == 0) {
+        sm[warp] = mb;
+        sb[warp] = wb;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t v = 0;
+        int b = 0;
+        for (int i = 0; i < nw; i++) {
+            v = max(v, sm[i]);
+            b |= sb[i];
+        }
+        p.part_max[blockIdx.x] = __uint_as_float(v);
+        p.part_bad[blockIdx.x] = b;
+        __threadfence();
+        atomicAdd(p.barrier, 1u);
+        unsigned spins = 0;
+        int timeout = 0;
+        while (ld_acquire_u32(p.barrier) < gridDim.x) {
+            if (++spins > kBarrierSpinLimit) {
+                timeout = 1;
+                break;
+            }
+            __nanosleep(64);
+        }
+        s_timeout = timeout;
+    }
+    __syncthreads();
+    if (s_timeout) {
+        if (threadIdx.x == 0 && p.status_dev) atomicOr(p.status_dev, 2);
+        return false;
+    }
+    uint32_t v = 0;
+    int b = 0;
+    for (int i = threadIdx.x; i < (int)gridDim.x; i += blockDim.x) {
+        v = max(v, __float_as_uint(__ldcg(p.part_max + i)));
+        b |= __ldcg(p.part_bad + i);
+    }
+    v = __reduce_max_sync(0xffffffffu, v);
+    b = __reduce_or_sync(0xffffffffu, (unsigned)b);
+    __syncthreads();
+    if (lane == 0) {
+        sm[warp] = v;
+        sb[warp] = b;
+    }
+    __syncthreads();
+    uint32_t amaxb = 0;
+    int anyb = 0;
+    for (int i = 0; i < nw; i++) {
+        amaxb = max(amaxb, sm[i]);
+        anyb |= sb[i];
+    }
+    S_out = __fdiv_rn(__uint_as_float(amaxb), __fmul_rn(6.0f, p.fp8_div));
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        p.S_out[0] = S_out;
+        if (anyb && p.status_dev) atomicOr(p.status_dev, 1);
+    }
+    return true;
+}
+
+// FIX = 1: default window (fixed length, unrolled, poison-padded table).
+// DYN = 1: the global scale is computed in this launch (see dynamic_scale).
+template <int DT, int METHOD, int OBJ, int BLOCK, int FIX, int DYN>
+__global__ void __launch_bounds__(256, NVFP4_QMINB) quantize_kernel(QuantParams p) {
+    constexpr int SEGS = BLOCK / 16;
+    constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
+    constexpr int FIX_K = 7 - FIX_LO + 1;
+    __shared__ Cand tab[kTabN];
+    build_table(tab);
+    __syncthreads();
+
+    float S;
+    if (DYN) {
+        if (!dynamic_scale<DT>(p, S)) return;
+    } else {
+        S = __ldg(p.S);
+    }
+    const float E = __frcp_rn(S);
+    const bool usable = (S > 0.0f) && isfinite(S) && isfinite(E);
+    const int lane = threadIdx.x & 31;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t nseg_pad = (p.nseg + 31) & ~(int64_t)31;
+
+    int64_t base = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31);
+    Raw cur;
+    if (base + lane < p.nseg) load_raw<DT>(p.x, base + lane, cur);
+
+    for (; base < nseg_pad; base += stride) {
+        const int64_t g = base + lane;
+        const bool valid = g < p.nseg;
+        Raw nxt;
+        if (g + stride < p.nseg) load_raw<DT>(p.x, g + stride, nxt);
+
+        float xv[16];
+        if (valid) {
+            raw_to_float<DT>(cur, xv);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 16; i++) xv[i] = 0.0f;
+        }
+        cur = nxt;
+
+        const int64_t blk = g / SEGS;               // scale-block index
+        int64_t row = 0, kbi = 0;
+        if (p.need_rowcol) {
+            if (p.narrow) {
+                const uint32_t b32 = (uint32_t)blk;
+                const uint32_t r32 = fast_div(b32, p.kb_div);
+                row = r32;
+                kbi = b32 - r32 * (uint32_t)p.kb;
+            } else {
+                row = blk / p.kb;
+                kbi = blk - row * p.kb;
+            }
+        }
+
+        u64 y2[8];
+        float m = 0.0f;
+#pragma unroll
+        for (int j = 0; j < 8; j++) {
+            const float a = usable ? __fmul_rn(xv[2 * j], E) : xv[2 * j];
+            const float b = usable ? __fmul_rn(xv[2 * j + 1], E) : xv[2 * j + 1];
+            m = fmaxf(m, fmaxf(fabsf(a), fabsf(b)));
+            y2[j] = pack2(a, b);
+        }
+        m = group_max<SEGS>(m);
+
+        u64 w2[8];
+        if (OBJ == 1) {
+            const int64_t col = kbi * BLOCK + (int64_t)(g % SEGS) * 16;
+            const float* wp = p.w + row * p.w_row_stride + col;
+            if (valid) {
+#pragma unroll
+                for (int j = 0; j < 4; j++) {
+                    const uint4 a = ld_ro16(wp + 4 * j);
+                    w2[2 * j] = pack2(__uint_as_float(a.x), __uint_as_float(a.y));
+                    w2[2 * j + 1] = pack2(__uint_as_float(a.z), __uint_as_float(a.w));
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < 8; j++) w2[j] = 0ull;
+            }
+        }
+
+        const bool zero = !usable || !(m > 0.0f);
+        float best = __int_as_float(0x7f800000);
+        int bestc = 0;
+        if (METHOD == 0) {
+            const float sbase = __fdiv_rn(m, 6.0f);
+            const int I0 = e4m3_floor_code(sbase);
+            if (FIX) {
+                const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
+                int bk = 0;
+#pragma unroll kCandUnroll
+                for (int k = 0; k < FIX_K; k++) {
+                    const Cand cd = tb[k];
+                    const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));
+                    if (L < best) {
+                        best = L;
+                        bk = k;
+                    }
+                }
+                bestc = I0 + FIX_LO + bk;
+            } else {
+                const int clo = min(max(I0 + p.win_lo, 1), 126);
+                const int chi = min(max(I0 + p.win_hi, 1), 126);
+                const int n = zero ? 0 : chi - clo + 1;
+                const int nmax = __reduce_max_sync(0xffffffffu, (unsigned)n);
+                bestc = clo;
+                for (int k = 0; k < nmax; k++) {
+                    const int c = min(clo + k, chi);    // repeats of chi never win the strict "<"
+                    const Cand cd = tab[c + kTabOff];
+                    const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));
+                    if (L < best) {
+                        best = L;
+                        bestc = c;
+                    }
+                }
+            }
+        } else {
+            const float sbase = __fdiv_rn(m, 6.0f);
+            const int c6 = max((int)e4m3_rn_code(sbase), 1);
+            bestc = c6;
+            if (METHOD == 2) {
+                const int c4 = max((int)e4m3_rn_code(__fdiv_rn(m, 4.0f)), 1);
+                const Cand d6 = tab[c6 + kTabOff], d4 = tab[c4 + kTabOff];
+                const float L6 = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, d6.r, (uint16_t)d6.nv));
+                const float L4 = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, d4.r, (uint16_t)d4.nv));
+                best = L6;
+                if (L4 < L6) {
+                    best = L4;
+                    bestc = c4;
+                }
+            } else if (p.block_loss) {
+                const Cand d6 = tab[c6 + kTabOff];
+                best = group_sum<SEGS>(seg_loss<0>(y2, w2, d6.r, (uint16_t)d6.nv));
+            }
+        }
+
+        // Emit packed nibbles for this thread's 16 elements.
+        uint32_t packed[2];
+        if (zero) {
+#pragma unroll
+            for (int h = 0; h < 2; h++) {
+                uint32_t acc = 0;
+#pragma unroll
+                for (int j = 0; j < 4; j++) {
+                    float a, b;
+                    unpack2(y2[4 * h + j], a, b);
+                    const uint32_t byte = (signbit(a) ? 0x08u : 0u) | (signbit(b) ? 0x80u : 0u);
+                    acc |= byte << (8 * j);
+                }
+                packed[h] = acc;
+            }
+            bestc = 0;
+            best = 0.0f;
+            if (p.block_loss) {
+                float s = 0.0f;
+#pragma unroll
+                for (int j = 0; j < 8; j++) {
+                    float a, b;
+                    unpack2(y2[j], a, b);
+                    if (OBJ == 1) {
+                        float wa, wb;
+                        unpack2(w2[j], wa, wb);
+                        s = __fmaf_rn(__fmul_rn(wa, a), a, s);
+                        s = __fmaf_rn(__fmul_rn(wb, b), b, s);
+                    } else {
+                        s = __fmaf_rn(a, a, s);
+                        s = __fmaf_rn(b, b, s);
+                    }
+                }
+                best = group_sum<SEGS>(s);
+            }
+        } else {
+            const float r = tab[bestc + kTabOff].r;
+            const u64 r2 = pack2(r, r);
+#pragma unroll
+            for (int h = 0; h < 2; h++) {
+                uint32_t acc = 0;
+#pragma unroll
+                for (int j = 0; j < 4; j++) {
+                    float a, b;
+                    unpack2(mul2(y2[4 * h + j], r2), a, b);
+                    acc |= e2m1x2(a, b) << (8 * j);
+                }
+                packed[h] = acc;
+            }
+        }
+
+        if (valid) {
+            *reinterpret_cast<uint2*>(p.codes + g * 8) = make_uint2(packed[0], packed[1]);
+            if ((g % SEGS) == 0) {
+                if (p.sf_linear) p.sf_linear[blk] = (uint8_t)bestc;
+                if (p.sf_swizzled) p.sf_swizzled[swizzle_offset(row, kbi, p.kpad4)] = (uint8_t)bestc;
+                if (p.block_loss) p.block_loss[blk] = best;
+            }
+        }
+    }
+}
+
+
+}  // namespace nvfp4

@@ -27,8 +27,8 @@ def L():
 def test_header_declares_the_api():
     assert declared_functions() == sorted([
         "nvfp4_status_string", "nvfp4_global_scale_workspace", "nvfp4_global_scale", "nvfp4_global_scale_noalloc",
-        "scalesweep_quantize",
-        "absmax_quantize", "four_over_six_quantize", "nvfp4_dequantize"])
+        "scalesweep_quantize", "absmax_quantize", "four_over_six_quantize", "nvfp4_dequantize",
+        "nvfp4_dynamic_workspace", "scalesweep_quantize_dynamic", "absmax_quantize_dynamic"])
 
 
 def test_library_exports_every_declared_symbol(L):
