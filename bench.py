@@ -589,6 +589,66 @@ def run_table7(args):
         print(json.dumps(res), flush=True)
 
 
+def run_quality(args):
+    """Quantisation error of AbsMax, 4/6, ScaleSweep, the FP8-quantised optimal
+    scale and the optimal FP32 scale (Appendix C) on synthetic 72B-shaped Laplace
+    weights -- the analogue of the paper's Fig. 1 (block sizes 16/32/64, MSE and
+    WMSE) and Fig. 2 (global scale divisor D).  NMSE = sum w (x - x_hat)^2 /
+    sum w x^2 over the sampled rows; gap = NMSE / NMSE(optimal FP32) - 1."""
+    from paper_2606_07618_gb300 import binding as B
+    from paper_2606_07618_gb300 import workloads as W
+    dev = "cuda"
+    wl = W.workload("qwen72b-b16-mse")
+    xs = [W.draw(t, rows=slice(0, args.quality_rows)).to(dev) for t in wl.tensors]
+    ws_ = [W.draw_weights(t).to(dev) for t in wl.tensors]
+    win = (B.NVFP4_WINDOW_DEFAULT, B.NVFP4_WINDOW_DEFAULT)
+
+    def study(block, obj, D):
+        num = {k: 0.0 for k in ("absmax", "four_six", "scalesweep", "fp8_opt", "fp32_opt")}
+        den = 0.0
+        for x, w in zip(xs, ws_):
+            rows, cols = x.shape
+            S = torch.empty(1, device=dev)
+            wsp = torch.empty(B.nvfp4_global_scale_workspace(x.numel()), dtype=torch.uint8, device=dev)
+            B.nvfp4_global_scale(x, D, S, None, wsp)
+            wt = w if obj else None
+            wf = (w.double() if obj else torch.ones(cols, dtype=torch.float64, device=dev))
+            xd = x.double()
+            den += float((xd * xd * wf).sum())
+            o = B.empty_outputs(rows, cols, block, device=dev, linear=True)
+            deq = torch.empty(rows, cols, device=dev)
+            for name in ("absmax", "four_six", "scalesweep"):
+                if name == "absmax":
+                    B.absmax_quantize(x, block, S, o["codes"], o["sf_linear"])
+                elif name == "four_six":
+                    B.four_over_six_quantize(x, block, S, obj, wt, 0, o["codes"], o["sf_linear"])
+                else:
+                    B.scalesweep_quantize(x, block, S, obj, wt, 0, *win, o["codes"], o["sf_linear"])
+                B.nvfp4_dequantize(o["codes"], o["sf_linear"], B.NVFP4_SF_LINEAR, S, rows, cols, block, deq)
+                num[name] += float(((xd - deq.double()) ** 2 * wf).sum())
+            nb = rows * cols // block
+            so, lo = torch.empty(nb, device=dev), torch.empty(nb, device=dev)
+            code, lf = torch.empty(nb, dtype=torch.uint8, device=dev), torch.empty(nb, device=dev)
+            B.nvfp4_optimal_scale(x, block, S, obj, wt, 0, so, lo, code, lf)
+            s2 = float(S.item()) ** 2
+            num["fp32_opt"] += float(lo.double().sum()) * s2
+            num["fp8_opt"] += float(lf.double().sum()) * s2
+        nm = {k: v / den for k, v in num.items()}
+        gap = {k: round(nm[k] / nm["fp32_opt"] - 1.0, 5) for k in nm if k != "fp32_opt"}
+        return {"block": block, "objective": "wmse" if obj else "mse", "D": D,
+                "nmse": {k: float(f"{v:.6g}") for k, v in nm.items()}, "gap_vs_fp32_opt": gap}
+
+    out = []
+    for block in (16, 32, 64):
+        for obj in (0, 1):
+            out.append(study(block, obj, 256.0))
+            print(json.dumps(out[-1]), flush=True)
+    for D in (448.0, 384.0, 192.0, 128.0, 64.0):
+        out.append(study(16, 0, D))
+        print(json.dumps(out[-1]), flush=True)
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -607,7 +667,12 @@ def main():
     ap.add_argument("--block", type=int, default=16)
     ap.add_argument("--reps", type=int, default=5)
     ap.add_argument("--table7", action="store_true")
+    ap.add_argument("--quality", action="store_true")
+    ap.add_argument("--quality-rows", type=int, default=2048)
     args = ap.parse_args()
+    if args.quality:
+        run_quality(args)
+        return
     if args.table7:
         run_table7(args)
         return

@@ -194,6 +194,23 @@ nvfp4_status four_over_six_quantize(const void* x, nvfp4_dtype dt, int64_t rows,
                                     float* block_loss, void* stream);
 
 /*
+ * Optimal real-valued block scale (Appendix C) and the FP8-quantised optimal
+ * scale (Appendix C, second paragraph), per block, in the S-normalised domain
+ * (y = fl(x * fl(1/S))): s_opt minimises sum w_i (y_i - s RN_E2M1(y_i/s))^2
+ * over real s > 0 by enumerating the quadratic segments between the
+ * breakpoints |y_i| / mu (mu the E2M1 midpoints); loss_opt is that minimum
+ * (fp32).  fp8_code (optional) is the better of floor_E4M3(s_opt) and
+ * ceil_E4M3(s_opt) under the sweep's arithmetic contract (ties to the floor),
+ * loss_fp8 (optional, needs fp8_code) its loss.  An analysis entry point: it
+ * measures the gap of any FP8 scale choice to the best FP32 scale.
+ *   x, S, obj, w, w_row_stride as scalesweep_quantize (4-byte alignment);
+ *   s_opt, loss_opt, loss_fp8: [rows*cols/block] float; fp8_code [rows*cols/block].
+ */
+nvfp4_status nvfp4_optimal_scale(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                                 const float* S, nvfp4_objective obj, const float* w, int64_t w_row_stride,
+                                 float* s_opt, float* loss_opt, uint8_t* fp8_code, float* loss_fp8, void* stream);
+
+/*
  * Dequantisation x_hat = fl32(fl32(q * s) * S) (Sec. 3.2 reconstruction; the
  * simulated quantisation of Sec. 5.1), written as fp32 or as the RNE bf16 of
  * that fp32 value.

@@ -58,9 +58,10 @@ def lib() -> ctypes.CDLL:
         L.nvfp4_dynamic_workspace.argtypes, L.nvfp4_dynamic_workspace.restype = [], sz
         L.scalesweep_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, i, p, i64, i, i, p, p, p, sz, p, p, p, p, p]
         L.absmax_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, p, p, p, sz, p, p, p, p, p]
+        L.nvfp4_optimal_scale.argtypes = [p, i, i64, i64, i, p, i, p, i64, p, p, p, p, p]
         for fn in ("nvfp4_global_scale", "nvfp4_global_scale_noalloc", "scalesweep_quantize", "absmax_quantize",
                    "four_over_six_quantize", "nvfp4_dequantize", "scalesweep_quantize_dynamic",
-                   "absmax_quantize_dynamic"):
+                   "absmax_quantize_dynamic", "nvfp4_optimal_scale"):
             getattr(L, fn).restype = i
         _lib = L
     return _lib
@@ -167,6 +168,15 @@ def absmax_quantize_dynamic(x, block: int, fp8_div: float, S_out, status, worksp
                                        _ptr(status), _ptr(workspace), ws_bytes, _ptr(codes), _ptr(sf_linear),
                                        _ptr(sf_swizzled), _ptr(block_loss), _stream(stream))
     _check("absmax_quantize_dynamic", rc)
+
+
+def nvfp4_optimal_scale(x, block: int, S, objective: int, w, w_row_stride: int, s_opt, loss_opt, fp8_code=None,
+                        loss_fp8=None, stream=None):
+    rows, cols = x.shape
+    rc = lib().nvfp4_optimal_scale(_ptr(x), _dtype(x), rows, cols, int(block), _ptr(S), int(objective), _ptr(w),
+                                   int(w_row_stride), _ptr(s_opt), _ptr(loss_opt), _ptr(fp8_code), _ptr(loss_fp8),
+                                   _stream(stream))
+    _check("nvfp4_optimal_scale", rc)
 
 
 def nvfp4_dequantize(codes, sf, layout: int, S, rows: int, cols: int, block: int, out, stream=None):

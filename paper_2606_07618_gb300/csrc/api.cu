@@ -281,6 +281,54 @@ nvfp4_status four_over_six_quantize(const void* x, nvfp4_dtype dt, int64_t rows,
                            block_loss, stream);
 }
 
+nvfp4_status nvfp4_optimal_scale(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
+                                 const float* S, nvfp4_objective obj, const float* w, int64_t w_row_stride,
+                                 float* s_opt, float* loss_opt, uint8_t* fp8_code, float* loss_fp8, void* stream) {
+    if (dt != NVFP4_IN_BF16 && dt != NVFP4_IN_F32) return NVFP4_ERR_INVALID_ARG;
+    if (obj != NVFP4_OBJ_MSE && obj != NVFP4_OBJ_WMSE) return NVFP4_ERR_INVALID_ARG;
+    Shape sh;
+    nvfp4_status st = check_shape(rows, cols, block, &sh);
+    if (st != NVFP4_OK) return st;
+    if (sh.n == 0) return NVFP4_OK;
+    if (!x || !S || !s_opt || !loss_opt || (loss_fp8 && !fp8_code)) return NVFP4_ERR_INVALID_ARG;
+    if (obj == NVFP4_OBJ_WMSE && (!w || (w_row_stride != 0 && w_row_stride < cols) || w_row_stride < 0))
+        return NVFP4_ERR_INVALID_ARG;
+    if (!aligned(x, 4) || !aligned(S, 4) || !aligned(s_opt, 4) || !aligned(loss_opt, 4) ||
+        (loss_fp8 && !aligned(loss_fp8, 4)) || (w && !aligned(w, 4)))
+        return NVFP4_ERR_ALIGNMENT;
+    const int64_t xbytes = sh.n * (dt == NVFP4_IN_BF16 ? 2 : 4);
+    const void* outs[4] = {s_opt, loss_opt, fp8_code, loss_fp8};
+    const int64_t olen[4] = {sh.nblocks * 4, sh.nblocks * 4, sh.nblocks, sh.nblocks * 4};
+    for (int i = 0; i < 4; i++) {
+        if (!outs[i]) continue;
+        if (overlap(outs[i], olen[i], x, xbytes) || overlap(outs[i], olen[i], S, 4)) return NVFP4_ERR_INVALID_ARG;
+        for (int j = i + 1; j < 4; j++)
+            if (overlap(outs[i], olen[i], outs[j], olen[j])) return NVFP4_ERR_INVALID_ARG;
+    }
+    if (!device_accessible(x) || !device_accessible(S) || !device_accessible(s_opt) || !device_accessible(loss_opt) ||
+        !device_accessible(fp8_code) || !device_accessible(loss_fp8) ||
+        (obj == NVFP4_OBJ_WMSE && !device_accessible(w)))
+        return NVFP4_ERR_INVALID_ARG;
+    const int sms = sm_count();
+    if (sms <= 0) return NVFP4_ERR_CUDA;
+    OptParams p;
+    p.x = x;
+    p.S = S;
+    p.w = obj == NVFP4_OBJ_WMSE ? w : nullptr;
+    p.w_row_stride = w_row_stride;
+    p.rows = rows;
+    p.cols = cols;
+    p.kb = sh.kb;
+    p.nblocks = sh.nblocks;
+    p.s_opt = s_opt;
+    p.loss_opt = loss_opt;
+    p.fp8_code = fp8_code;
+    p.loss_fp8 = loss_fp8;
+    cudaError_t e = launch_optimal_scale(p, dt == NVFP4_IN_BF16 ? 0 : 1, obj == NVFP4_OBJ_WMSE ? 1 : 0, block, sms,
+                                         static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
+}
+
 nvfp4_status nvfp4_dequantize(const uint8_t* codes, const uint8_t* sf, nvfp4_sf_layout layout, const float* S,
                               int64_t rows, int64_t cols, int block, void* out, nvfp4_dtype out_dt,
                               void* stream) {

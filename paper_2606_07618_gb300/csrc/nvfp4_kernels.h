@@ -59,6 +59,19 @@ constexpr size_t kDynWorkspace = (size_t)kAmaxParts * 8 + 256;
 cudaError_t launch_global_scale_parts(const void* x, int dtype, int64_t n, float fp8_div, float* S_out,
                                       int* status_dev, float* part_max, int* part_bad, int grid, cudaStream_t s);
 
+struct OptParams {
+    const void* x;
+    const float* S;
+    const float* w;
+    int64_t w_row_stride;
+    int64_t rows, cols, kb, nblocks;
+    float* s_opt;
+    float* loss_opt;
+    uint8_t* fp8_code;
+    float* loss_fp8;
+};
+cudaError_t launch_optimal_scale(const OptParams& p, int dtype, int obj, int block, int sms, cudaStream_t s);
+
 struct DequantParams {
     const uint8_t* codes;
     const uint8_t* sf;

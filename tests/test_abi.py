@@ -28,7 +28,8 @@ def test_header_declares_the_api():
     assert declared_functions() == sorted([
         "nvfp4_status_string", "nvfp4_global_scale_workspace", "nvfp4_global_scale", "nvfp4_global_scale_noalloc",
         "scalesweep_quantize", "absmax_quantize", "four_over_six_quantize", "nvfp4_dequantize",
-        "nvfp4_dynamic_workspace", "scalesweep_quantize_dynamic", "absmax_quantize_dynamic"])
+        "nvfp4_dynamic_workspace", "scalesweep_quantize_dynamic", "absmax_quantize_dynamic",
+        "nvfp4_optimal_scale"])
 
 
 def test_library_exports_every_declared_symbol(L):
