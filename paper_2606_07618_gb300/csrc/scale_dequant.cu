@@ -147,16 +147,18 @@ cudaError_t launch_global_scale_parts(const void* x, int dtype, int64_t n, float
 }
 
 // ---------------------------------------------------------------------------
-// Dequantisation: one thread per 16-element segment.  q and s are decoded by
-// the native converts into f16, q*s is exact in f16 (at most 7 significant
-// bits, within range), then one fp32 multiply by S rounds once.
+// Dequantisation: each thread produces exactly one 16-byte store (8 bf16 or 4
+// fp32 outputs), so a warp writes 512 contiguous bytes per store instruction.
+// q and s are decoded by the native converts into f16, q*s is exact in f16 (at
+// most 7 significant bits, within range), then one fp32 multiply by S rounds once.
 template <int OUT_BF16>
 __global__ void __launch_bounds__(256) dequant_kernel(DequantParams p) {
+    constexpr int EPT = OUT_BF16 ? 8 : 4;          // elements per thread
     const float S = __ldg(p.S);
-    const int segs = p.block / 16;
+    const int64_t nchunk = p.nseg * (16 / EPT);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    auto scale_offset = [&](int64_t g) -> int64_t {
-        const int64_t blk = g / segs;
+    auto scale_offset = [&](int64_t e0) -> int64_t {
+        const int64_t blk = e0 / p.block;           // element index -> scale block
         if (!p.swizzled) return blk;
         int64_t row, kbi;
         if (p.narrow) {
@@ -169,57 +171,53 @@ __global__ void __launch_bounds__(256) dequant_kernel(DequantParams p) {
         }
         return swizzle_offset(row, kbi, p.kpad4);
     };
-    int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    uint2 c_next = make_uint2(0, 0);
+    auto load_codes = [&](int64_t c) -> uint32_t {
+        return EPT == 8 ? __ldg(reinterpret_cast<const uint32_t*>(p.codes) + c)
+                        : (uint32_t)__ldg(reinterpret_cast<const uint16_t*>(p.codes) + c);
+    };
+    int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    uint32_t cw_next = 0;
     uint8_t s_next = 0;
-    if (g < p.nseg) {
-        c_next = __ldg(reinterpret_cast<const uint2*>(p.codes + g * 8));
-        s_next = __ldg(p.sf + scale_offset(g));
+    if (c < nchunk) {
+        cw_next = load_codes(c);
+        s_next = __ldg(p.sf + scale_offset(c * EPT));
     }
-    for (; g < p.nseg; g += stride) {
-        const uint2 c = c_next;
+    for (; c < nchunk; c += stride) {
+        const uint32_t cw = cw_next;
         const uint8_t sc = s_next;
-        if (g + stride < p.nseg) {                 // prefetch the next segment
-            c_next = __ldg(reinterpret_cast<const uint2*>(p.codes + (g + stride) * 8));
-            s_next = __ldg(p.sf + scale_offset(g + stride));
+        if (c + stride < nchunk) {                 // prefetch the next chunk
+            cw_next = load_codes(c + stride);
+            s_next = __ldg(p.sf + scale_offset((c + stride) * EPT));
         }
-        const uint16_t vh = e4m3_to_f16bits(sc);
-        const uint32_t vv = (uint32_t)vh * 0x10001u;
-        const uint32_t cw[2] = {c.x, c.y};
-        float out[16];
+        const uint32_t vv = (uint32_t)e4m3_to_f16bits(sc) * 0x10001u;
+        float out[EPT];
 #pragma unroll
-        for (int h = 0; h < 2; h++) {
-#pragma unroll
-            for (int j = 0; j < 4; j++) {
-                uint32_t q2, prod;
-                const uint16_t byte = (uint16_t)((cw[h] >> (8 * j)) & 0xFFu);
-                asm("{\n\t.reg .b8 b;\n\tcvt.u8.u16 b, %1;\n\tcvt.rn.f16x2.e2m1x2 %0, b;\n\t}" : "=r"(q2) : "h"(byte));
-                asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(prod) : "r"(q2), "r"(vv));
-                out[8 * h + 2 * j] = __fmul_rn(f16bits_to_f32((uint16_t)(prod & 0xFFFF)), S);
-                out[8 * h + 2 * j + 1] = __fmul_rn(f16bits_to_f32((uint16_t)(prod >> 16)), S);
-            }
+        for (int j = 0; j < EPT / 2; j++) {
+            uint32_t q2, prod;
+            const uint16_t byte = (uint16_t)((cw >> (8 * j)) & 0xFFu);
+            asm("{\n\t.reg .b8 b;\n\tcvt.u8.u16 b, %1;\n\tcvt.rn.f16x2.e2m1x2 %0, b;\n\t}" : "=r"(q2) : "h"(byte));
+            asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(prod) : "r"(q2), "r"(vv));
+            out[2 * j] = __fmul_rn(f16bits_to_f32((uint16_t)(prod & 0xFFFF)), S);
+            out[2 * j + 1] = __fmul_rn(f16bits_to_f32((uint16_t)(prod >> 16)), S);
         }
         if (OUT_BF16) {
-            uint32_t o[8];
+            uint32_t o[4];
 #pragma unroll
-            for (int j = 0; j < 8; j++) {
-                __nv_bfloat16 a = __float2bfloat16_rn(out[2 * j]), b = __float2bfloat16_rn(out[2 * j + 1]);
+            for (int j = 0; j < 4; j++) {
+                const __nv_bfloat16 a = __float2bfloat16_rn(out[2 * j]), b = __float2bfloat16_rn(out[2 * j + 1]);
                 o[j] = (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(b) << 16);
             }
-            uint4* op = reinterpret_cast<uint4*>(static_cast<char*>(p.out) + g * 32);
-            op[0] = make_uint4(o[0], o[1], o[2], o[3]);
-            op[1] = make_uint4(o[4], o[5], o[6], o[7]);
+            reinterpret_cast<uint4*>(p.out)[c] = make_uint4(o[0], o[1], o[2], o[3]);
         } else {
-            float4* op = reinterpret_cast<float4*>(static_cast<char*>(p.out) + g * 64);
-#pragma unroll
-            for (int j = 0; j < 4; j++) op[j] = make_float4(out[4 * j], out[4 * j + 1], out[4 * j + 2], out[4 * j + 3]);
+            reinterpret_cast<float4*>(p.out)[c] = make_float4(out[0], out[1], out[2], out[3]);
         }
     }
 }
 
 cudaError_t launch_dequantize(const DequantParams& p, int out_dtype, int sms, cudaStream_t s) {
     if (p.nseg <= 0) return cudaSuccess;
-    int64_t grid = (p.nseg + 255) / 256;
+    const int64_t nchunk = p.nseg * (out_dtype == 0 ? 2 : 4);
+    int64_t grid = (nchunk + 255) / 256;
     if (grid > (int64_t)sms * 8) grid = (int64_t)sms * 8;
     if (out_dtype == 0)
         dequant_kernel<1><<<(int)grid, 256, 0, s>>>(p);
