@@ -17,7 +17,8 @@
 // fma.f32.f16 (exact product q*(-v), one rounding) -> fma.f32x2 accumulate.
 //
 // Candidate table: entry code+128 holds {fl(1/v_c), f16 bits of -v_c} for codes
-// 1..126 and a poison entry {+inf, -inf} elsewhere.  A poison candidate's loss
+// 1..126 and a poison entry {+inf, -inf} elsewhere.  (8-byte entries measured
+// faster than 16-byte ones holding the packed {r, r} operand.)  A poison candidate's loss
 // is inf or NaN, so it never wins the strict "<" -- this lets the default
 // windows run a fixed, fully unrolled loop over [I0+lo, I0+hi] with no clamping
 // (those windows always contain a real code).  Custom windows clamp instead.
@@ -69,21 +70,33 @@ __device__ __forceinline__ void load_raw(const void* x, int64_t g, Raw& r) {
     }
 }
 
+// The segment's 16 inputs as 8 packed pairs y = fl(x*E) (one f32x2 multiply
+// per pair) and the block max m = max |y|.
 template <int DT>
-__device__ __forceinline__ void raw_to_float(const Raw& r, float (&xv)[16]) {
+__device__ __forceinline__ float raw_to_y(const Raw& r, u64 E2, u64 (&y2)[8]) {
+    uint32_t u[16];
     if (DT == 0) {
-        const uint32_t u[8] = {r.a.x, r.a.y, r.a.z, r.a.w, r.b.x, r.b.y, r.b.z, r.b.w};
+        const uint32_t p[8] = {r.a.x, r.a.y, r.a.z, r.a.w, r.b.x, r.b.y, r.b.z, r.b.w};
 #pragma unroll
         for (int j = 0; j < 8; j++) {
-            xv[2 * j] = bf16lo(u[j]);
-            xv[2 * j + 1] = bf16hi(u[j]);
+            u[2 * j] = p[j] << 16;
+            u[2 * j + 1] = p[j] & 0xFFFF0000u;
         }
     } else {
-        const uint32_t u[16] = {r.a.x, r.a.y, r.a.z, r.a.w, r.b.x, r.b.y, r.b.z, r.b.w,
+        const uint32_t p[16] = {r.a.x, r.a.y, r.a.z, r.a.w, r.b.x, r.b.y, r.b.z, r.b.w,
                                 r.c.x, r.c.y, r.c.z, r.c.w, r.d.x, r.d.y, r.d.z, r.d.w};
 #pragma unroll
-        for (int j = 0; j < 16; j++) xv[j] = __uint_as_float(u[j]);
+        for (int j = 0; j < 16; j++) u[j] = p[j];
     }
+    float m = 0.0f;
+#pragma unroll
+    for (int j = 0; j < 8; j++) {
+        y2[j] = mul2(pack2(__uint_as_float(u[2 * j]), __uint_as_float(u[2 * j + 1])), E2);
+        float a, b;
+        unpack2(y2[j], a, b);
+        m = fmaxf(m, fmaxf(fabsf(a), fabsf(b)));
+    }
+    return m;
 }
 
 // Loss of one candidate on this thread's 16 elements.
@@ -261,8 +274,10 @@ __global__ void __launch_bounds__(256, NVFP4_QMINB) quantize_kernel(QuantParams 
     } else {
         S = __ldg(p.S);
     }
-    const float E = __frcp_rn(S);
+    float E = __frcp_rn(S);
     const bool usable = (S > 0.0f) && isfinite(S) && isfinite(E);
+    if (!usable) E = 1.0f;                          // y = x: only signs (and sum w x^2) are emitted
+    const u64 E2 = pack2(E, E);
     const int lane = threadIdx.x & 31;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     const int64_t nseg_pad = (p.nseg + 31) & ~(int64_t)31;
@@ -277,13 +292,15 @@ __global__ void __launch_bounds__(256, NVFP4_QMINB) quantize_kernel(QuantParams 
         Raw nxt;
         if (g + stride < p.nseg) load_raw<DT>(p.x, g + stride, nxt);
 
-        float xv[16];
+        u64 y2[8];
+        float m = 0.0f;
         if (valid) {
-            raw_to_float<DT>(cur, xv);
+            m = raw_to_y<DT>(cur, E2, y2);
         } else {
 #pragma unroll
-            for (int i = 0; i < 16; i++) xv[i] = 0.0f;
+            for (int j = 0; j < 8; j++) y2[j] = 0ull;
         }
+        m = group_max<SEGS>(m);
         cur = nxt;
 
         const int64_t blk = g / SEGS;               // scale-block index
@@ -300,16 +317,6 @@ __global__ void __launch_bounds__(256, NVFP4_QMINB) quantize_kernel(QuantParams 
             }
         }
 
-        u64 y2[8];
-        float m = 0.0f;
-#pragma unroll
-        for (int j = 0; j < 8; j++) {
-            const float a = usable ? __fmul_rn(xv[2 * j], E) : xv[2 * j];
-            const float b = usable ? __fmul_rn(xv[2 * j + 1], E) : xv[2 * j + 1];
-            m = fmaxf(m, fmaxf(fabsf(a), fabsf(b)));
-            y2[j] = pack2(a, b);
-        }
-        m = group_max<SEGS>(m);
 
         u64 w2[8];
         if (OBJ == 1) {
@@ -423,14 +430,14 @@ __global__ void __launch_bounds__(256, NVFP4_QMINB) quantize_kernel(QuantParams 
             const u64 r2 = pack2(r, r);
 #pragma unroll
             for (int h = 0; h < 2; h++) {
-                uint32_t acc = 0;
+                uint32_t b[4];
 #pragma unroll
                 for (int j = 0; j < 4; j++) {
-                    float a, b;
-                    unpack2(mul2(y2[4 * h + j], r2), a, b);
-                    acc |= e2m1x2(a, b) << (8 * j);
+                    float lo, hi;
+                    unpack2(mul2(y2[4 * h + j], r2), lo, hi);
+                    b[j] = e2m1x2(lo, hi);
                 }
-                packed[h] = acc;
+                packed[h] = b[0] | (b[1] << 8) | (b[2] << 16) | (b[3] << 24);
             }
         }
 
