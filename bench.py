@@ -569,6 +569,7 @@ def run_table7(args):
             return f
 
         res = {"batch": b}
+        reps = 50
         for kind in ("absmax", "mse", "wmse", "absmax_dyn", "mse_dyn", "wmse_dyn", "absmax_fused", "mse_fused",
                      "wmse_fused"):
             f = op(kind)
@@ -576,13 +577,40 @@ def run_table7(args):
                 f()
             torch.cuda.synchronize()
             a, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            reps = 50
             a.record()
             for _ in range(reps):
                 f()
             e.record()
             torch.cuda.synchronize()
             res[kind + "_ms"] = round(a.elapsed_time(e) / reps, 4)
+        # The same calls captured once in a CUDA graph and replayed: the library
+        # never allocates or synchronises, so a caller can remove the per-call
+        # host cost this way; what remains is the device time per call.
+        for kind in ("absmax", "mse", "wmse", "mse_dyn", "wmse_dyn"):
+            f = op(kind)
+            try:
+                side = torch.cuda.Stream()
+                side.wait_stream(torch.cuda.current_stream())
+                with torch.cuda.stream(side):
+                    for _ in range(3):
+                        f()
+                torch.cuda.current_stream().wait_stream(side)
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    for _ in range(reps):
+                        f()
+                g.replay()
+                torch.cuda.synchronize()
+                a, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record()
+                for _ in range(4):
+                    g.replay()
+                e.record()
+                torch.cuda.synchronize()
+                res[kind + "_graph_ms"] = round(a.elapsed_time(e) / (4 * reps), 4)
+            except RuntimeError as exc:          # capture refused: report, keep the eager numbers
+                res[kind + "_graph_ms"] = None
+                res[kind + "_graph_error"] = str(exc)[:120]
         res["mse_rel"] = round(res["mse_ms"] / res["absmax_ms"], 3)
         res["wmse_rel"] = round(res["wmse_ms"] / res["absmax_ms"], 3)
         rows.append(res)

@@ -70,6 +70,12 @@ __device__ __forceinline__ void load_raw(const void* x, int64_t g, Raw& r) {
     }
 }
 
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
 // The segment's 16 inputs as 8 packed pairs y = fl(x*E) (one f32x2 multiply
 // per pair) and the block max m = max |y|.
 template <int DT>
@@ -88,15 +94,19 @@ __device__ __forceinline__ float raw_to_y(const Raw& r, u64 E2, u64 (&y2)[8]) {
 #pragma unroll
         for (int j = 0; j < 16; j++) u[j] = p[j];
     }
-    float m = 0.0f;
+    float av[16];
 #pragma unroll
     for (int j = 0; j < 8; j++) {
         y2[j] = mul2(pack2(__uint_as_float(u[2 * j]), __uint_as_float(u[2 * j + 1])), E2);
         float a, b;
         unpack2(y2[j], a, b);
-        m = fmaxf(m, fmaxf(fabsf(a), fabsf(b)));
+        av[2 * j] = fabsf(a);
+        av[2 * j + 1] = fabsf(b);
     }
-    return m;
+    // three-input max tree (NaNs are skipped, as by fmaxf)
+    const float p0 = max3f(av[0], av[1], av[2]), p1 = max3f(av[3], av[4], av[5]), p2 = max3f(av[6], av[7], av[8]);
+    const float p3 = max3f(av[9], av[10], av[11]), p4 = max3f(av[12], av[13], av[14]);
+    return max3f(max3f(p0, p1, p2), max3f(p3, p4, av[15]), 0.0f);
 }
 
 // Loss of one candidate on this thread's 16 elements.
