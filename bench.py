@@ -677,6 +677,81 @@ def run_quality(args):
     return out
 
 
+def run_ldlq(args):
+    """LDLQ (GPTQ with ScaleSweep scales, static reordering; Appendix A.2) on the
+    Llama-3-8B layer shapes: the Hessian factorization per input width and the
+    error-feedback pass per weight, CUDA-event timed, with the proxy loss
+    tr(E H E^T) of LDLQ vs rounding at the same scales on sampled rows.
+    Synthetic Hessians: low-rank (256) plus diagonal with lognormal channel
+    scales (sigma 0.8), built with torch matmul outside the timed region."""
+    from paper_2606_07618_gb300 import binding as B
+    dev = "cuda"
+    g = torch.Generator().manual_seed(23)
+    hess = {}
+    rows_out = []
+    for n in (4096, 14336):
+        scale = torch.exp(torch.randn(n, generator=g) * 0.8).to(dev)
+        A = torch.randn(n, 256, generator=g).to(dev) * scale[:, None]
+        H = (A @ A.T) / 256 + torch.diag(scale * scale * 0.05)
+        perm = torch.empty(n, dtype=torch.int32, device=dev)
+        U = torch.empty(n, n, device=dev)
+        D = torch.empty(n, device=dev)
+        st = torch.zeros(1, dtype=torch.int32, device=dev)
+        ws = torch.empty(B.nvfp4_ldlq_prepare_workspace(n), dtype=torch.uint8, device=dev)
+        B.nvfp4_ldlq_prepare(H, 0.01, perm, U, D, st, ws)
+        torch.cuda.synchronize()
+        a, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = max(1, args.reps // 2)
+        a.record()
+        for _ in range(reps):
+            B.nvfp4_ldlq_prepare(H, 0.01, perm, U, D, st, ws)
+        e.record()
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(e) / reps
+        hess[n] = (H, perm, U)
+        rows_out.append({"ldlq_prepare": n, "ms": round(ms, 3), "status": int(st.item()),
+                         "tflops_fp32": round(2 * n ** 3 / 3 / (ms * 1e-3) / 1e12, 2)})
+        print(json.dumps(rows_out[-1]), flush=True)
+    for name, (rows, cols) in (("q", (4096, 4096)), ("k", (1024, 4096)), ("gate", (14336, 4096)),
+                               ("down", (4096, 14336))):
+        H, perm, U = hess[cols]
+        W = (torch.randn(rows, cols, generator=g) * 0.02).to(torch.bfloat16).to(dev)
+        S = torch.empty(1, device=dev)
+        gws = torch.empty(B.nvfp4_global_scale_workspace(W.numel()), dtype=torch.uint8, device=dev)
+        B.nvfp4_global_scale(W, 256.0, S, None, gws)
+        sf = torch.empty(rows, cols // 16, dtype=torch.uint8, device=dev)
+        rtn = torch.empty(rows, cols // 2, dtype=torch.uint8, device=dev)
+        imp = torch.diagonal(H).contiguous()
+        B.scalesweep_quantize(W, 16, S, B.NVFP4_OBJ_WMSE, imp, 0, B.NVFP4_WINDOW_DEFAULT, B.NVFP4_WINDOW_DEFAULT,
+                              rtn, sf)
+        codes = torch.empty_like(rtn)
+        st = torch.zeros(1, dtype=torch.int32, device=dev)
+        ws = torch.empty(B.nvfp4_ldlq_workspace(rows, cols), dtype=torch.uint8, device=dev)
+        B.ldlq_quantize(W, 16, S, sf, perm, U, codes, st, ws)
+        torch.cuda.synchronize()
+        a, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = max(1, args.reps // 2)
+        a.record()
+        for _ in range(reps):
+            B.ldlq_quantize(W, 16, S, sf, perm, U, codes, st, ws)
+        e.record()
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(e) / reps
+        # proxy loss on 256 sampled rows (evaluation only)
+        idx = torch.linspace(0, rows - 1, 256, device=dev).long()
+        losses = []
+        for c in (codes, rtn):
+            xh = torch.empty(256, cols, device=dev)
+            B.nvfp4_dequantize(c[idx].contiguous(), sf[idx].contiguous(), B.NVFP4_SF_LINEAR, S, 256, cols, 16, xh)
+            E = W[idx].float() - xh
+            losses.append(float(((E @ H) * E).sum()))
+        rows_out.append({"ldlq_quantize": name, "rows": rows, "cols": cols, "ms": round(ms, 3),
+                         "status": int(st.item()), "gemm_tflops_fp32": round(rows * cols * cols / (ms * 1e-3) / 1e12, 2),
+                         "proxy_loss_ldlq_over_rtn": round(losses[0] / losses[1], 4)})
+        print(json.dumps(rows_out[-1]), flush=True)
+    return rows_out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -697,7 +772,11 @@ def main():
     ap.add_argument("--table7", action="store_true")
     ap.add_argument("--quality", action="store_true")
     ap.add_argument("--quality-rows", type=int, default=2048)
+    ap.add_argument("--ldlq", action="store_true")
     args = ap.parse_args()
+    if args.ldlq:
+        run_ldlq(args)
+        return
     if args.quality:
         run_quality(args)
         return

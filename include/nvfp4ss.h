@@ -222,6 +222,53 @@ nvfp4_status nvfp4_dequantize(const uint8_t* codes, const uint8_t* sf, nvfp4_sf_
                               int64_t rows, int64_t cols, int block, void* out, nvfp4_dtype out_dt,
                               void* stream);
 
+/*
+ * LDLQ / GPTQ with ScaleSweep block scales (Appendix A.2, "GPTQ" paragraph):
+ * GPTQ's error-feedback pass in QuIP's LDLQ form, damping damp * mean(diag H)
+ * (the paper uses damp = 0.01), and static reordering -- the block scales are
+ * fixed beforehand (e.g. by scalesweep_quantize with WMSE weights diag(H)) and
+ * the input channels are processed in descending order of diag(H).
+ *
+ * nvfp4_ldlq_prepare factors the Hessian once per weight matrix:
+ *   H       [n, n] float, the input Gram matrix X^T X (any positive scaling),
+ *           symmetric; every entry H[perm[i], perm[j]] is read.  4-byte aligned.
+ *   perm    [n] int32 out: perm[k] = original column processed k-th (diagonal
+ *           descending, ties by ascending index, NaN last).
+ *   U       [n, n] float out (4-byte aligned, must not overlap H): the strictly
+ *           upper factor of H_pi + lambda I = (U + I) diag(D) (U + I)^T in
+ *           processing order (zeros on and below the diagonal).  Also used as
+ *           the factorization's scratch.
+ *   D       [n] float out.
+ *   status_dev  optional int on the device: |= 4 if the damped Hessian is not
+ *           positive definite or has a non-finite diagonal (a failing pivot is
+ *           replaced by 1 so the outputs stay finite, but they are not a
+ *           factorization then).
+ *   workspace   device bytes, at least nvfp4_ldlq_prepare_workspace(n).
+ * Cost: n^3/3 fp32 multiply-adds (blocked Cholesky, 64-wide panels).
+ */
+size_t nvfp4_ldlq_prepare_workspace(int64_t n);
+nvfp4_status nvfp4_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* perm, float* U, float* D,
+                                int* status_dev, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * ldlq_quantize: W [rows, cols] (bf16 or f32, original column order) to packed
+ * NVFP4 codes [rows, cols/2] (original order) with the fixed scales sf_linear
+ * [rows, cols/block] (E4M3 codes, linear layout) and global scale S (device).
+ * Column k of the processing order gets T_k = W_k + sum_{i<k} (W_i - What_i)
+ * U_ik, What_k = Q(T_k), with Q the sweep's fp32 rounding at the fixed scale:
+ * y = fl(T*E), q = RNE_E2M1(fl(y*fl(1/v))), What = fl(fl(q*v)*S); a zero scale
+ * code or an unusable S quantizes to signed zeros, an exactly zero y to +0.
+ *   perm, U from nvfp4_ldlq_prepare (cols = n); status_dev optional: |= 8 if
+ *   perm holds an index outside [0, cols) (the entry is then read as 0).
+ *   workspace   device bytes, at least nvfp4_ldlq_workspace(rows, cols):
+ *           rows*cols*5 + rows*256 + cols*4 plus alignment.
+ * Cost: rows*cols^2/2 fp32 multiply-adds; rows are independent.
+ */
+size_t nvfp4_ldlq_workspace(int64_t rows, int64_t cols);
+nvfp4_status ldlq_quantize(const void* W, nvfp4_dtype dt, int64_t rows, int64_t cols, int block, const float* S,
+                           const uint8_t* sf_linear, const int32_t* perm, const float* U, uint8_t* codes,
+                           int* status_dev, void* workspace, size_t ws_bytes, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

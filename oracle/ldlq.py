@@ -24,7 +24,9 @@ Q is NVFP4 rounding with the fixed block scale of the element's (original)
 block, taken in the kernels' float32 contract: t = fl32(T), y = fl32(t*E) with
 E = fl32(1/S), q = RNE_E2M1(fl32(y*fl32(1/v))) (saturating at 6, ties to the even
 code), What = fl32(fl32(q*v)*S).  A block whose scale code is 0, or an unusable
-global scale, quantizes to signed zeros (the sweep's zero rule).
+global scale, quantizes to signed zeros (the sweep's zero rule).  A target that
+is exactly zero takes the +0 code: the sign of a zero sum depends on the
+summation order, which neither side fixes (reading; LDLQ itself is silent).
 
 The same result in GPTQ's own form (error feedback through the upper Cholesky
 factor of the inverse Hessian) is ``gptq``; the two are independent
@@ -58,10 +60,12 @@ def rne_e2m1(a):
     return np.where(a >= 6.0, 7, k).astype(np.int64)
 
 
-def quantize_fixed(t, S, code):
+def quantize_fixed(t, S, code, zero_positive=False):
     """Q(t) with fixed E4M3 scale codes: returns (nibbles, dequantized values).
 
-    t: float64 targets; code: per-element scale codes (0..126)."""
+    t: float64 targets; code: per-element scale codes (0..126); zero_positive:
+    an exactly zero y takes the +0 code (LDLQ targets), else its own sign (the
+    sweep's rounding of inputs)."""
     t32 = np.asarray(t, dtype=np.float64).astype(np.float32)
     S32 = np.float32(S)
     with np.errstate(divide="ignore", over="ignore", invalid="ignore"):
@@ -70,6 +74,8 @@ def quantize_fixed(t, S, code):
     code = np.asarray(code, dtype=np.int64)
     y = (t32 * E).astype(np.float32) if usable else t32
     sign = np.signbit(y)
+    if zero_positive:
+        sign = sign & (y != 0)
     zero = (code == 0) | (not usable)
     v = e4m3_value(np.where(zero, 1, code)).astype(np.float32)
     r = (np.float32(1.0) / v).astype(np.float32)
@@ -124,7 +130,7 @@ def ldlq(W, H, S, sf, block=16, alpha=0.01):
     T = np.zeros((m, n))
     for k in range(n):
         T[:, k] = Wp[:, k] + (Wp[:, :k] - What[:, :k]) @ U[:k, k]
-        nib[:, k], What[:, k] = quantize_fixed(T[:, k], S, code_el[:, k])
+        nib[:, k], What[:, k] = quantize_fixed(T[:, k], S, code_el[:, k], zero_positive=True)
     inv = np.empty(n, dtype=np.int64)
     inv[perm] = np.arange(n)
     return {"nib": nib[:, inv], "What": What[:, inv], "perm": perm, "U": U, "D": D, "T": T}
@@ -143,7 +149,7 @@ def gptq(W, H, S, sf, block=16, alpha=0.01):
     What = np.zeros((m, n))
     nib = np.zeros((m, n), dtype=np.int64)
     for i in range(n):
-        nib[:, i], What[:, i] = quantize_fixed(Wt[:, i], S, code_el[:, i])
+        nib[:, i], What[:, i] = quantize_fixed(Wt[:, i], S, code_el[:, i], zero_positive=True)
         err = (Wt[:, i] - What[:, i]) / R[i, i]
         Wt[:, i + 1:] -= np.outer(err, R[i, i + 1:])
     inv = np.empty(n, dtype=np.int64)
@@ -171,8 +177,9 @@ def decision_margin(T, S, code):
     boundary (midpoint), relative to max(1, value): small margins are where a
     float32 and a float64 accumulation of T may round differently."""
     t32 = np.asarray(T, dtype=np.float64).astype(np.float32)
-    E = np.float32(1.0) / np.float32(S)
-    v = e4m3_value(np.where(np.asarray(code) == 0, 1, code)).astype(np.float32)
-    z = np.abs(((t32 * E).astype(np.float32) * (np.float32(1.0) / v)).astype(np.float32)).astype(np.float64)
-    mids = np.array([0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0])
-    return np.min(np.abs(z[..., None] - mids), axis=-1) / np.maximum(1.0, z)
+    with np.errstate(divide="ignore", over="ignore", invalid="ignore"):
+        E = np.float32(1.0) / np.float32(S)
+        v = e4m3_value(np.where(np.asarray(code) == 0, 1, code)).astype(np.float32)
+        z = np.abs(((t32 * E).astype(np.float32) * (np.float32(1.0) / v)).astype(np.float32)).astype(np.float64)
+        mids = np.array([0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0])
+        return np.min(np.abs(z[..., None] - mids), axis=-1) / np.maximum(1.0, z)

@@ -59,9 +59,13 @@ def lib() -> ctypes.CDLL:
         L.scalesweep_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, i, p, i64, i, i, p, p, p, sz, p, p, p, p, p]
         L.absmax_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, p, p, p, sz, p, p, p, p, p]
         L.nvfp4_optimal_scale.argtypes = [p, i, i64, i64, i, p, i, p, i64, p, p, p, p, p]
+        L.nvfp4_ldlq_prepare_workspace.argtypes, L.nvfp4_ldlq_prepare_workspace.restype = [i64], sz
+        L.nvfp4_ldlq_prepare.argtypes = [p, i64, f, p, p, p, p, p, sz, p]
+        L.nvfp4_ldlq_workspace.argtypes, L.nvfp4_ldlq_workspace.restype = [i64, i64], sz
+        L.ldlq_quantize.argtypes = [p, i, i64, i64, i, p, p, p, p, p, p, p, sz, p]
         for fn in ("nvfp4_global_scale", "nvfp4_global_scale_noalloc", "scalesweep_quantize", "absmax_quantize",
                    "four_over_six_quantize", "nvfp4_dequantize", "scalesweep_quantize_dynamic",
-                   "absmax_quantize_dynamic", "nvfp4_optimal_scale"):
+                   "absmax_quantize_dynamic", "nvfp4_optimal_scale", "nvfp4_ldlq_prepare", "ldlq_quantize"):
             getattr(L, fn).restype = i
         _lib = L
     return _lib
@@ -200,3 +204,31 @@ def empty_outputs(rows: int, cols: int, block: int, device="cuda", linear=True, 
         if swizzled else None
     out["block_loss"] = torch.empty(rows * (cols // block), dtype=torch.float32, device=device) if loss else None
     return out
+
+
+def nvfp4_ldlq_prepare_workspace(n: int) -> int:
+    return int(lib().nvfp4_ldlq_prepare_workspace(int(n)))
+
+
+def nvfp4_ldlq_prepare(H, damp: float, perm, U, D, status=None, workspace=None, stream=None):
+    """Damped, reordered UDU^T factor of the Hessian H [n, n] float32 for LDLQ:
+    perm [n] int32, U [n, n] float32, D [n] float32 (outputs)."""
+    n = H.shape[0]
+    ws_bytes = workspace.numel() * workspace.element_size()
+    rc = lib().nvfp4_ldlq_prepare(_ptr(H), n, float(damp), _ptr(perm), _ptr(U), _ptr(D), _ptr(status),
+                                  _ptr(workspace), ws_bytes, _stream(stream))
+    _check("nvfp4_ldlq_prepare", rc)
+
+
+def nvfp4_ldlq_workspace(rows: int, cols: int) -> int:
+    return int(lib().nvfp4_ldlq_workspace(int(rows), int(cols)))
+
+
+def ldlq_quantize(W, block: int, S, sf_linear, perm, U, codes, status=None, workspace=None, stream=None):
+    """LDLQ (GPTQ) quantization of W [rows, cols] with the fixed scales sf_linear,
+    processing order perm and factor U from nvfp4_ldlq_prepare."""
+    rows, cols = W.shape
+    ws_bytes = workspace.numel() * workspace.element_size()
+    rc = lib().ldlq_quantize(_ptr(W), _dtype(W), rows, cols, int(block), _ptr(S), _ptr(sf_linear), _ptr(perm),
+                             _ptr(U), _ptr(codes), _ptr(status), _ptr(workspace), ws_bytes, _stream(stream))
+    _check("ldlq_quantize", rc)

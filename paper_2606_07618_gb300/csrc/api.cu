@@ -3,6 +3,7 @@
 // library never allocates, frees or synchronises; every call is asynchronous on
 // the caller's stream.
 #include <climits>
+#include <cmath>
 #include <cstdint>
 #include <cstring>
 
@@ -363,6 +364,85 @@ nvfp4_status nvfp4_dequantize(const uint8_t* codes, const uint8_t* sf, nvfp4_sf_
     p.block = block;
     p.out = out;
     cudaError_t e = launch_dequantize(p, out_dt == NVFP4_IN_BF16 ? 0 : 1, sms, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
+}
+
+size_t nvfp4_ldlq_prepare_workspace(int64_t n) { return n > 0 ? ldlq_prepare_workspace(n) : 0; }
+
+nvfp4_status nvfp4_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* perm, float* U, float* D,
+                                int* status_dev, void* workspace, size_t ws_bytes, void* stream) {
+    if (n < 0 || !(damp >= 0.0f) || !isfinite(damp)) return NVFP4_ERR_INVALID_ARG;
+    if (n == 0) return NVFP4_OK;
+    if (n > (int64_t)1 << 20) return NVFP4_ERR_RANGE;
+    if (!H || !perm || !U || !D || !workspace) return NVFP4_ERR_INVALID_ARG;
+    if (ws_bytes < ldlq_prepare_workspace(n)) return NVFP4_ERR_INVALID_ARG;
+    if (!aligned(H, 4) || !aligned(perm, 4) || !aligned(U, 4) || !aligned(D, 4) || !aligned(workspace, 256) ||
+        (status_dev && !aligned(status_dev, 4)))
+        return NVFP4_ERR_ALIGNMENT;
+    const int64_t mat = n * n * 4;
+    const void* bufs[6] = {H, perm, U, D, workspace, status_dev};
+    const int64_t lens[6] = {mat, n * 4, mat, n * 4, (int64_t)ldlq_prepare_workspace(n), 4};
+    for (int i = 0; i < 6; i++)
+        for (int j = i + 1; j < 6; j++)
+            if (overlap(bufs[i], lens[i], bufs[j], lens[j])) return NVFP4_ERR_INVALID_ARG;
+    for (int i = 0; i < 6; i++)
+        if (!device_accessible(bufs[i])) return NVFP4_ERR_INVALID_ARG;
+    const int sms = sm_count();
+    if (sms <= 0) return NVFP4_ERR_CUDA;
+    cudaError_t e = launch_ldlq_prepare(H, n, damp, perm, U, D, status_dev, workspace, sms,
+                                        static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
+}
+
+size_t nvfp4_ldlq_workspace(int64_t rows, int64_t cols) {
+    int64_t rc;
+    if (rows <= 0 || cols <= 0 || !mul_ok(rows, cols, &rc) || rc > INT64_MAX / 8) return 0;
+    return ldlq_quantize_workspace(rows, cols);
+}
+
+nvfp4_status ldlq_quantize(const void* W, nvfp4_dtype dt, int64_t rows, int64_t cols, int block, const float* S,
+                           const uint8_t* sf_linear, const int32_t* perm, const float* U, uint8_t* codes,
+                           int* status_dev, void* workspace, size_t ws_bytes, void* stream) {
+    if (dt != NVFP4_IN_BF16 && dt != NVFP4_IN_F32) return NVFP4_ERR_INVALID_ARG;
+    Shape sh;
+    nvfp4_status st = check_shape(rows, cols, block, &sh);
+    if (st != NVFP4_OK) return st;
+    if (sh.n == 0) return NVFP4_OK;
+    if (cols > (int64_t)1 << 20 || rows > (int64_t)1 << 23) return NVFP4_ERR_RANGE;
+    if (!W || !S || !sf_linear || !perm || !U || !codes || !workspace) return NVFP4_ERR_INVALID_ARG;
+    if (ws_bytes < ldlq_quantize_workspace(rows, cols)) return NVFP4_ERR_INVALID_ARG;
+    if (!aligned(W, dt == NVFP4_IN_BF16 ? 2 : 4) || !aligned(S, 4) || !aligned(perm, 4) || !aligned(U, 4) ||
+        !aligned(workspace, 256) || (status_dev && !aligned(status_dev, 4)))
+        return NVFP4_ERR_ALIGNMENT;
+    const int64_t wbytes = sh.n * (dt == NVFP4_IN_BF16 ? 2 : 4);
+    const void* ins[6] = {W, S, sf_linear, perm, U, status_dev};
+    const int64_t ilen[6] = {wbytes, 4, sh.nblocks, cols * 4, cols * cols * 4, 4};
+    const int64_t wsb = (int64_t)ldlq_quantize_workspace(rows, cols);
+    for (int i = 0; i < 6; i++)
+        if (overlap(codes, sh.n / 2, ins[i], ilen[i]) || overlap(workspace, wsb, ins[i], ilen[i]))
+            return NVFP4_ERR_INVALID_ARG;
+    if (overlap(codes, sh.n / 2, workspace, wsb)) return NVFP4_ERR_INVALID_ARG;
+    for (int i = 0; i < 6; i++)
+        if (!device_accessible(ins[i])) return NVFP4_ERR_INVALID_ARG;
+    if (!device_accessible(codes) || !device_accessible(workspace)) return NVFP4_ERR_INVALID_ARG;
+    const int sms = sm_count();
+    if (sms <= 0) return NVFP4_ERR_CUDA;
+    LdlqParams p;
+    p.W = W;
+    p.rows = rows;
+    p.n = cols;
+    p.perm = perm;
+    p.U = U;
+    p.sf = sf_linear;
+    p.kb = sh.kb;
+    p.block = block;
+    p.S = S;
+    p.status = status_dev;
+    p.T = nullptr;
+    p.qb = nullptr;
+    p.Ep = nullptr;
+    cudaError_t e = launch_ldlq_quantize(p, dt == NVFP4_IN_BF16 ? 0 : 1, codes, workspace, sms,
+                                         static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
 }
 

@@ -29,7 +29,8 @@ def test_header_declares_the_api():
         "nvfp4_status_string", "nvfp4_global_scale_workspace", "nvfp4_global_scale", "nvfp4_global_scale_noalloc",
         "scalesweep_quantize", "absmax_quantize", "four_over_six_quantize", "nvfp4_dequantize",
         "nvfp4_dynamic_workspace", "scalesweep_quantize_dynamic", "absmax_quantize_dynamic",
-        "nvfp4_optimal_scale"])
+        "nvfp4_optimal_scale", "nvfp4_ldlq_prepare_workspace", "nvfp4_ldlq_prepare", "nvfp4_ldlq_workspace",
+        "ldlq_quantize"])
 
 
 def test_library_exports_every_declared_symbol(L):
@@ -80,3 +81,35 @@ def test_validation_without_gpu(L):
     assert L.nvfp4_dequantize(FAKE, FAKE + 4096, 2, FAKE + 8192, 4, 64, 32, FAKE + 16384, 1, None) == 2
     assert L.nvfp4_dequantize(FAKE, FAKE + 4096, 3, FAKE + 8192, 4, 64, 16, FAKE + 16384, 1, None) == 1
     assert L.nvfp4_dequantize(FAKE, FAKE + 4096, 1, FAKE + 8192, 4, 64, 16, FAKE + 8, 1, None) == 3
+
+
+def test_ldlq_validation_without_gpu(L):
+    f = ctypes.c_float
+    ws = 1 << 24
+    prep = lambda H=FAKE, n=64, damp=0.01, perm=FAKE + 0x100000, U=FAKE + 0x200000, D=FAKE + 0x300000, \
+        wsp=FAKE + 0x400000, wsb=ws: L.nvfp4_ldlq_prepare(H, n, f(damp), perm, U, D, None, wsp, wsb, None)
+    assert prep(n=-1) == 1
+    assert prep(damp=-1.0) == 1
+    assert prep(damp=float("nan")) == 1
+    assert prep(n=0) == 0                             # nothing to do, no launch
+    assert prep(n=(1 << 20) + 1) == 4
+    assert prep(U=None) == 1
+    assert prep(wsb=16) == 1                          # workspace too small
+    assert prep(H=FAKE + 2) == 3
+    assert prep(U=FAKE + 0x8000) == 1                 # U overlaps H (64*64*4 bytes)
+    assert L.nvfp4_ldlq_prepare_workspace(4096) >= 4096 * 4
+    assert L.nvfp4_ldlq_workspace(4096, 4096) >= 4096 * 4096 * 5
+    assert L.nvfp4_ldlq_workspace(-1, 64) == 0
+    q = lambda W=FAKE, dt=0, rows=4, cols=64, block=16, S=FAKE + 0x100000, sf=FAKE + 0x110000, \
+        perm=FAKE + 0x120000, U=FAKE + 0x130000, codes=FAKE + 0x200000, wsp=FAKE + 0x400000, wsb=ws: \
+        L.ldlq_quantize(W, dt, rows, cols, block, S, sf, perm, U, codes, None, wsp, wsb, None)
+    assert q(block=8) == 2
+    assert q(cols=40) == 1
+    assert q(dt=5) == 1
+    assert q(rows=0) == 0
+    assert q(perm=None) == 1
+    assert q(wsb=64) == 1
+    assert q(W=FAKE + 1) == 3
+    assert q(codes=FAKE) == 1                         # codes overlap W
+    assert q(wsp=FAKE + 0x130000) == 1                # workspace overlaps U
+

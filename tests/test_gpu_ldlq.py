@@ -1,0 +1,206 @@
+"""LDLQ (GPTQ) with fixed ScaleSweep scales on the GPU against the oracle.
+
+* Prepare: the processing order is bit-exact; the fp32 UDU^T factor matches the
+  oracle's float64 one to fp32 accuracy and reproduces the damped, reordered
+  Hessian (backward error).
+* Quantize: LDLQ is a sequential fixed point, What_k = Q(T_k(What_<k)), so one
+  float32-vs-float64 flip near a rounding boundary changes every later target a
+  little.  The element-by-element check therefore recomputes each GPU decision
+  in float64 from the GPU's own earlier decisions and factor -- T = W_pi +
+  (W_pi - What_pi) U -- and requires the GPU nibble to equal Q(T) wherever T is
+  not within float32 accumulation error of a rounding boundary.  The first
+  processed column has no feedback and must match exactly; a diagonal Hessian
+  must give plain rounding at the fixed scales, bit for bit; the proxy loss must
+  match the oracle's own LDLQ and beat rounding.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import ldlq as L
+from test_oracle_ldlq import fixed_scales, rand_problem
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+MARGIN = 2e-5          # relative distance to an E2M1 midpoint treated as a tie
+
+
+@pytest.fixture(scope="module")
+def B():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_07618_gb300 import binding
+    binding.lib()
+    oracle.build()
+    return binding
+
+
+def prepare(B, H, damp=0.01):
+    n = H.shape[0]
+    Hd = torch.as_tensor(np.ascontiguousarray(H), dtype=torch.float32).to(DEV)
+    perm = torch.empty(n, dtype=torch.int32, device=DEV)
+    U = torch.empty(n, n, dtype=torch.float32, device=DEV)
+    D = torch.empty(n, dtype=torch.float32, device=DEV)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    ws = torch.empty(B.nvfp4_ldlq_prepare_workspace(n), dtype=torch.uint8, device=DEV)
+    B.nvfp4_ldlq_prepare(Hd, damp, perm, U, D, st, ws)
+    torch.cuda.synchronize()
+    return perm, U, D, int(st.item())
+
+
+def quantize(B, W, S, sf, perm, U, block=16):
+    rows, cols = W.shape
+    codes = torch.empty(rows, cols // 2, dtype=torch.uint8, device=DEV)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    ws = torch.empty(B.nvfp4_ldlq_workspace(rows, cols), dtype=torch.uint8, device=DEV)
+    Sd = torch.tensor([S], dtype=torch.float32, device=DEV)
+    sfd = torch.as_tensor(np.ascontiguousarray(sf), dtype=torch.uint8).to(DEV)
+    B.ldlq_quantize(W, block, Sd, sfd, perm, U, codes, st, ws)
+    torch.cuda.synchronize()
+    return codes.cpu().numpy(), int(st.item())
+
+
+def unpack(codes):
+    return np.stack([codes & 0xF, codes >> 4], axis=-1).reshape(codes.shape[0], -1).astype(np.int64)
+
+
+def conditional_parity(W, S, sf, block, perm, U, codes):
+    """Returns (mismatches outside the tie margin, exempted mismatches, elements)."""
+    rows, cols = W.shape
+    nib = unpack(codes)
+    What = oracle.dequantize(codes, sf, oracle.LAYOUT_LINEAR, S, rows, cols, block).astype(np.float64)
+    T = L.targets(W, What, perm, U)
+    code_el = np.asarray(sf, dtype=np.int64)[:, perm // block]
+    ref, _ = L.quantize_fixed(T, S, code_el, zero_positive=True)
+    got = nib[:, perm]
+    diff = ref != got
+    tie = L.decision_margin(T, S, code_el) < MARGIN
+    tiny = np.abs(T) <= 1e-6 * np.abs(W).max()             # sign of a near-zero target (zero scales)
+    exempt = tie | (tiny & ((code_el == 0) | ((ref & 7) == 0)))
+    return int(np.sum(diff & ~exempt)), int(np.sum(diff & exempt)), diff.size, diff[:, 0].sum()
+
+
+@pytest.mark.parametrize("n", [16, 64, 100, 200, 257])
+def test_prepare_matches_oracle(B, n):
+    _, H = rand_problem(2, n, n)
+    H = H.astype(np.float32).astype(np.float64)
+    np.fill_diagonal(H, np.round(np.diag(H), 1) + 0.5)     # repeated diagonal values: the order's tie rule
+    perm, U, D, st = prepare(B, H)
+    assert st == 0
+    Hd, perm_ref = L.damp_and_order(H)
+    assert np.array_equal(perm.cpu().numpy(), perm_ref)
+    Hp = Hd[np.ix_(perm_ref, perm_ref)]
+    U_ref, D_ref = L.udu(Hp)
+    Ug, Dg = U.double().cpu().numpy(), D.double().cpu().numpy()
+    assert np.all(np.tril(Ug) == 0)
+    assert np.allclose(Dg, D_ref, rtol=2e-4)
+    assert np.abs(Ug - U_ref).max() <= 2e-4 * max(1.0, np.abs(U_ref).max())
+    I = np.eye(n)
+    R = (Ug + I) @ np.diag(Dg) @ (Ug + I).T - Hp
+    assert np.abs(R).max() <= 2e-5 * np.abs(Hp).max()
+
+
+def test_diagonal_hessian_is_rounding(B):
+    rng = np.random.default_rng(3)
+    W = (rng.standard_normal((33, 208)) * 0.02).astype(np.float32)
+    H = np.diag(np.exp(rng.standard_normal(208))).astype(np.float32).astype(np.float64)
+    S, sf = fixed_scales(W.astype(np.float64), H)
+    perm, U, D, st = prepare(B, H)
+    assert st == 0 and torch.count_nonzero(U).item() == 0
+    codes, st = quantize(B, torch.from_numpy(W).to(DEV), S, sf, perm, U)
+    assert st == 0
+    _, ref = oracle.block_losses_at(W, 16, S, sf, want_codes=True)
+    assert np.array_equal(codes, ref)
+
+
+@pytest.mark.parametrize("rows,cols,block", [(1, 64, 16), (64, 256, 16), (37, 208, 16), (48, 192, 32),
+                                             (16, 320, 64)])
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_ldlq_conditional_parity_small(B, rows, cols, block, dtype):
+    W64, H = rand_problem(rows, cols, rows * 7 + cols)
+    Wt = torch.from_numpy(W64.astype(np.float32)).to(dtype)
+    W = Wt.float().numpy().astype(np.float64)
+    H = H.astype(np.float32).astype(np.float64)
+    S, sf = fixed_scales(W, H, block)
+    perm, U, D, st = prepare(B, H)
+    assert st == 0
+    codes, st = quantize(B, Wt.to(DEV), S, sf, perm, U, block)
+    assert st == 0
+    bad, exempt, total, first = conditional_parity(W, S, sf, block, perm.cpu().numpy().astype(np.int64),
+                                                   U.double().cpu().numpy(), codes)
+    assert bad == 0 and first == 0
+    assert exempt <= max(2, total // 200)
+    # quality: the oracle's own float64 LDLQ, and rounding at the same scales
+    What = oracle.dequantize(codes, sf, oracle.LAYOUT_LINEAR, S, rows, cols, block).astype(np.float64)
+    ref = L.ldlq(W, H, S, sf, block)
+    rtn = L.quantize_fixed(W, S, np.repeat(sf, block, axis=1))[1]
+    lg, lo, lr = (L.proxy_loss(W, x, H) for x in (What, ref["What"], rtn))
+    assert lg == pytest.approx(lo, rel=0.02 if rows >= 16 else 0.1)
+    if rows >= 16:
+        assert lg < lr
+
+
+def test_ldlq_full_size_sampled_rows(B):
+    """A 4096 x 4096 weight (q/o projection shape) with a low-rank-plus-diagonal
+    Hessian of heavy-tailed channel scales; 48 sampled rows checked in float64."""
+    n, rows = 4096, 4096
+    g = torch.Generator().manual_seed(17)
+    scale = torch.exp(torch.randn(n, generator=g) * 0.8)
+    A = torch.randn(n, 192, generator=g, dtype=torch.float64) * scale[:, None].double()
+    H = (A @ A.T / 192 + torch.diag(scale.double() ** 2 * 0.05)).float().double().numpy()
+    W = (torch.randn(rows, n, generator=g) * 0.02).to(torch.bfloat16)
+    Wn = W.float().numpy().astype(np.float64)
+    S, _ = oracle.global_scale(Wn.astype(np.float32), 256.0)
+    Sd = torch.tensor([S], dtype=torch.float32, device=DEV)
+    sf = torch.empty(rows, n // 16, dtype=torch.uint8, device=DEV)
+    codes0 = torch.empty(rows, n // 2, dtype=torch.uint8, device=DEV)
+    imp = torch.from_numpy(np.diag(H).astype(np.float32)).to(DEV)
+    B.scalesweep_quantize(W.to(DEV), 16, Sd, B.NVFP4_OBJ_WMSE, imp, 0, B.NVFP4_WINDOW_DEFAULT,
+                          B.NVFP4_WINDOW_DEFAULT, codes0, sf)
+    perm, U, D, st = prepare(B, H)
+    assert st == 0
+    sfn = sf.cpu().numpy()
+    codes, st = quantize(B, W.to(DEV), S, sfn, perm, U)
+    assert st == 0
+    idx = np.unique(np.linspace(0, rows - 1, 48).astype(np.int64))
+    bad, exempt, total, first = conditional_parity(Wn[idx], S, sfn[idx], 16, perm.cpu().numpy().astype(np.int64),
+                                                   U.double().cpu().numpy(), codes[idx])
+    assert bad == 0 and first == 0
+    assert exempt <= total // 200
+    What = oracle.dequantize(codes[idx], sfn[idx], oracle.LAYOUT_LINEAR, S, len(idx), n, 16).astype(np.float64)
+    rtn = L.quantize_fixed(Wn[idx], S, np.repeat(sfn[idx], 16, axis=1))[1]
+    assert L.proxy_loss(Wn[idx], What, H) < 0.9 * L.proxy_loss(Wn[idx], rtn, H)
+
+
+def test_zero_scales_and_unusable_global_scale(B):
+    W64, H = rand_problem(8, 64, 5)
+    W = W64.astype(np.float32)
+    S, sf = fixed_scales(W64, H)
+    sf = sf.copy()
+    sf[1, :] = 0
+    sf[3, 2] = 0
+    perm, U, D, st = prepare(B, H)
+    for Sv in (S, 0.0):
+        codes, st = quantize(B, torch.from_numpy(W).to(DEV), Sv, sf, perm, U)
+        assert st == 0
+        bad, exempt, total, first = conditional_parity(W64, Sv, sf, 16, perm.cpu().numpy().astype(np.int64),
+                                                       U.double().cpu().numpy(), codes)
+        assert bad == 0 and first == 0
+    codes, st = quantize(B, torch.from_numpy(W).to(DEV), float("inf"), sf, perm, U)
+    assert st == 0 and not np.any(codes & 0x77)             # an unusable scale leaves signs only
+
+
+def test_failures_are_reported_not_faulted(B):
+    n = 64
+    perm, U, D, st = prepare(B, -np.eye(n))
+    assert st & 4                                           # not positive definite
+    Hn = np.eye(n)
+    Hn[5, 5] = np.nan
+    perm2, U2, D2, st2 = prepare(B, Hn)
+    assert st2 & 4 and sorted(perm2.cpu().numpy().tolist()) == list(range(n))
+    W = torch.randn(4, n, device=DEV)
+    bad_perm = perm.clone()
+    bad_perm[3] = n + 5
+    codes, st3 = quantize(B, W, 0.001, np.full((4, n // 16), 60, np.uint8), bad_perm, U)
+    assert st3 & 8

@@ -94,10 +94,10 @@ def test_two_column_feedback_closed_form():
     sf = np.full((3, 1), 56)                                  # one block, v = 1.0 (code 56)
     res = L.ldlq(W, H, 1.0, sf, block=2, alpha=0.0)
     assert list(res["perm"]) == [0, 1]
-    w0q = L.quantize_fixed(W[:, 0], 1.0, np.full(3, 56))[1]
+    w0q = L.quantize_fixed(W[:, 0], 1.0, np.full(3, 56), zero_positive=True)[1]
     t1 = W[:, 1] + (W[:, 0] - w0q) * (1.1 / 2.0)
     assert np.allclose(res["T"][:, 1], t1, rtol=1e-15)
-    assert np.array_equal(res["What"][:, 1], L.quantize_fixed(t1, 1.0, np.full(3, 56))[1])
+    assert np.array_equal(res["What"][:, 1], L.quantize_fixed(t1, 1.0, np.full(3, 56), zero_positive=True)[1])
 
 
 @pytest.mark.parametrize("seed", [4, 5, 6])
