@@ -689,7 +689,11 @@ def run_ldlq(args):
     g = torch.Generator().manual_seed(23)
     hess = {}
     rows_out = []
-    for n in (4096, 14336):
+    shapes = (("q", (4096, 4096)), ("k", (1024, 4096)), ("gate", (14336, 4096)), ("down", (4096, 14336)))
+    if args.ldlq_shape:
+        r_, c_ = (int(v) for v in args.ldlq_shape.split("x"))
+        shapes = (("custom", (r_, c_)),)
+    for n in sorted({c for _, (_, c) in shapes}):
         scale = torch.exp(torch.randn(n, generator=g) * 0.8).to(dev)
         A = torch.randn(n, 256, generator=g).to(dev) * scale[:, None]
         H = (A @ A.T) / 256 + torch.diag(scale * scale * 0.05)
@@ -712,8 +716,7 @@ def run_ldlq(args):
         rows_out.append({"ldlq_prepare": n, "ms": round(ms, 3), "status": int(st.item()),
                          "tflops_fp32": round(2 * n ** 3 / 3 / (ms * 1e-3) / 1e12, 2)})
         print(json.dumps(rows_out[-1]), flush=True)
-    for name, (rows, cols) in (("q", (4096, 4096)), ("k", (1024, 4096)), ("gate", (14336, 4096)),
-                               ("down", (4096, 14336))):
+    for name, (rows, cols) in shapes:
         H, perm, U = hess[cols]
         W = (torch.randn(rows, cols, generator=g) * 0.02).to(torch.bfloat16).to(dev)
         S = torch.empty(1, device=dev)
@@ -773,6 +776,7 @@ def main():
     ap.add_argument("--quality", action="store_true")
     ap.add_argument("--quality-rows", type=int, default=2048)
     ap.add_argument("--ldlq", action="store_true")
+    ap.add_argument("--ldlq-shape", default=None, help="one ROWSxCOLS weight instead of the Llama-3-8B shapes")
     args = ap.parse_args()
     if args.ldlq:
         run_ldlq(args)

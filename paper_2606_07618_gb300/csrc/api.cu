@@ -439,8 +439,9 @@ nvfp4_status ldlq_quantize(const void* W, nvfp4_dtype dt, int64_t rows, int64_t 
     p.S = S;
     p.status = status_dev;
     p.T = nullptr;
+    p.Wp = nullptr;
     p.qb = nullptr;
-    p.Ep = nullptr;
+    p.sfp = nullptr;
     cudaError_t e = launch_ldlq_quantize(p, dt == NVFP4_IN_BF16 ? 0 : 1, codes, workspace, sms,
                                          static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;

@@ -29,7 +29,7 @@ namespace nvfp4 {
 
 namespace {
 
-constexpr int kP = kLdlqPanel;        // 64
+constexpr int kP = 64;                // Cholesky panel width
 constexpr int kLd = 132;              // GEMM smem row stride (floats): 128 + 4, 16-byte rows
 
 inline int64_t imin64(int64_t a, int64_t b) { return a < b ? a : b; }
@@ -106,56 +106,115 @@ __global__ void __launch_bounds__(256) gather_h_kernel(const float* H, int64_t n
 }
 
 // Cholesky of the nb x nb diagonal block at k0 (lower, in place) and its inverse
-// (lower, 64 x 64 with zeros) into Linv.  A pivot that is not positive and finite
-// sets bit 4 of the status word and is replaced by 1 so the values stay finite.
+// (lower, 64 x 64) into Linv.  The block is padded to 64 with an identity; each
+// of the 256 threads keeps a 4 x 4 tile in registers.  The pivots stay
+// unscaled, A = M diag(p) M^T with M unit lower triangular: at column j the
+// threads holding column j publish it to shared memory (double-buffered, one
+// barrier per column) and every tile subtracts a_ij a_lj / p_j.  Then
+// L = M diag(sqrt p) and L^-1 = diag(1/sqrt p) M^-1, with M^-1 by forward
+// elimination in the same scheme (column k of M and row k of M^-1 published per
+// step).  A pivot that is not positive and finite sets bit 4 of the status word
+// and is replaced by 1 so the values stay finite.
 __global__ void __launch_bounds__(256) potrf_kernel(float* A, int64_t n, int64_t k0, int nb, float* Linv,
                                                     int* status) {
-    __shared__ float a[kP][kP + 1];
-    __shared__ float li[kP][kP + 1];
-    __shared__ int s_bad;
-    for (int e = threadIdx.x; e < kP * kP; e += blockDim.x) {
-        const int i = e / kP, j = e % kP;
-        a[i][j] = (i < nb && j < nb) ? A[(k0 + i) * n + k0 + j] : 0.0f;
-        li[i][j] = 0.0f;
-    }
-    if (threadIdx.x == 0) s_bad = 0;
-    __syncthreads();
-    for (int j = 0; j < nb; j++) {
-        if (threadIdx.x == 0) {
-            float p = a[j][j];
-            if (!(p > 0.0f) || !isfinite(p)) {
-                s_bad = 1;
-                p = 1.0f;
+    __shared__ __align__(16) float colv[2][kP];
+    __shared__ __align__(16) float rowv[2][kP];
+    __shared__ float piv[kP];
+    const int r0 = (threadIdx.x >> 4) * 4, c0 = (threadIdx.x & 15) * 4;
+    float t[4][4];
+#pragma unroll
+    for (int di = 0; di < 4; di++)
+#pragma unroll
+        for (int dl = 0; dl < 4; dl++) {
+            const int i = r0 + di, l = c0 + dl;
+            float v = (i < nb && l < nb && l <= i) ? A[(k0 + i) * n + k0 + l] : 0.0f;
+            if (i >= nb && i == l) v = 1.0f;
+            t[di][dl] = v;
+        }
+    int bad = 0;
+    for (int j = 0; j < kP; j++) {
+        const int b = j & 1;
+        if (c0 <= j && j < c0 + 4) {
+#pragma unroll
+            for (int di = 0; di < 4; di++) {
+                const int q = j - c0;
+                const float v = q == 0 ? t[di][0] : q == 1 ? t[di][1] : q == 2 ? t[di][2] : t[di][3];
+                colv[b][r0 + di] = v;
             }
-            a[j][j] = __fsqrt_rn(p);
         }
         __syncthreads();
-        const float dj = a[j][j];
-        for (int i = j + 1 + threadIdx.x; i < nb; i += blockDim.x) a[i][j] = __fdiv_rn(a[i][j], dj);
-        __syncthreads();
-        const int m = nb - j - 1;
-        for (int e = threadIdx.x; e < m * m; e += blockDim.x) {
-            const int i = j + 1 + e / m, l = j + 1 + e % m;
-            if (l <= i) a[i][l] = __fmaf_rn(-a[i][j], a[l][j], a[i][l]);
+        float p = colv[b][j];
+        if (!(p > 0.0f) || !isfinite(p)) {
+            bad = 1;
+            p = 1.0f;
         }
-        __syncthreads();
-    }
-    if (threadIdx.x < nb) {                       // column c of L^-1 by forward substitution
-        const int c = threadIdx.x;
-        li[c][c] = __fdiv_rn(1.0f, a[c][c]);
-        for (int i = c + 1; i < nb; i++) {
-            float s = 0.0f;
-            for (int l = c; l < i; l++) s = __fmaf_rn(a[i][l], li[l][c], s);
-            li[i][c] = __fdiv_rn(-s, a[i][i]);
+        if (threadIdx.x == 0) piv[j] = p;
+        const float ip = __frcp_rn(p);
+        const float4 ci = *reinterpret_cast<const float4*>(&colv[b][r0]);
+        const float4 cl = *reinterpret_cast<const float4*>(&colv[b][c0]);
+        const float civ[4] = {ci.x, ci.y, ci.z, ci.w}, clv[4] = {cl.x, cl.y, cl.z, cl.w};
+#pragma unroll
+        for (int di = 0; di < 4; di++) {
+            const int i = r0 + di;
+            const float aij = __fmul_rn(civ[di], ip);
+#pragma unroll
+            for (int dl = 0; dl < 4; dl++) {
+                const int l = c0 + dl;
+                if (i > j && l > j && l <= i) t[di][dl] = __fmaf_rn(-aij, clv[dl], t[di][dl]);
+            }
         }
     }
     __syncthreads();
-    for (int e = threadIdx.x; e < kP * kP; e += blockDim.x) {
-        const int i = e / kP, j = e % kP;
-        if (i < nb && j <= i) A[(k0 + i) * n + k0 + j] = a[i][j];
-        Linv[e] = li[i][j];
+    // M (strictly lower part) in the tiles: m_il = a_il / p_l
+#pragma unroll
+    for (int di = 0; di < 4; di++)
+#pragma unroll
+        for (int dl = 0; dl < 4; dl++)
+            if (c0 + dl < r0 + di) t[di][dl] = __fmul_rn(t[di][dl], __frcp_rn(piv[c0 + dl]));
+    // X = M^-1 (unit lower), tile x: row k of X is final at step k
+    float x[4][4];
+#pragma unroll
+    for (int di = 0; di < 4; di++)
+#pragma unroll
+        for (int dc = 0; dc < 4; dc++) x[di][dc] = (r0 + di == c0 + dc) ? 1.0f : 0.0f;
+    for (int k = 0; k < kP; k++) {
+        const int b = k & 1;
+        if (c0 <= k && k < c0 + 4) {                 // column k of M
+#pragma unroll
+            for (int di = 0; di < 4; di++) {
+                const int q = k - c0;
+                const float v = q == 0 ? t[di][0] : q == 1 ? t[di][1] : q == 2 ? t[di][2] : t[di][3];
+                colv[b][r0 + di] = v;
+            }
+        }
+        if (r0 <= k && k < r0 + 4) {                 // row k of X
+#pragma unroll
+            for (int dc = 0; dc < 4; dc++) {
+                const int q = k - r0;
+                const float v = q == 0 ? x[0][dc] : q == 1 ? x[1][dc] : q == 2 ? x[2][dc] : x[3][dc];
+                rowv[b][c0 + dc] = v;
+            }
+        }
+        __syncthreads();
+        const float4 mi = *reinterpret_cast<const float4*>(&colv[b][r0]);
+        const float4 xk = *reinterpret_cast<const float4*>(&rowv[b][c0]);
+        const float miv[4] = {mi.x, mi.y, mi.z, mi.w}, xkv[4] = {xk.x, xk.y, xk.z, xk.w};
+#pragma unroll
+        for (int di = 0; di < 4; di++)
+#pragma unroll
+            for (int dc = 0; dc < 4; dc++)
+                if (r0 + di > k && c0 + dc <= k) x[di][dc] = __fmaf_rn(-miv[di], xkv[dc], x[di][dc]);
     }
-    if (threadIdx.x == 0 && s_bad && status) atomicOr(status, 4);
+#pragma unroll
+    for (int di = 0; di < 4; di++)
+#pragma unroll
+        for (int dl = 0; dl < 4; dl++) {
+            const int i = r0 + di, l = c0 + dl;
+            const float sl = __fsqrt_rn(piv[l]);
+            if (i < nb && l <= i) A[(k0 + i) * n + k0 + l] = i == l ? sl : __fmul_rn(t[di][dl], sl);
+            Linv[i * kP + l] = l <= i ? __fmul_rn(x[di][dl], __frsqrt_rn(piv[i])) : 0.0f;
+        }
+    if (threadIdx.x == 0 && bad && status) atomicOr(status, 4);
 }
 
 // Panel below the diagonal block: rows i >= k0+nb, X = A_panel * Linv^T (one warp per row).
@@ -182,53 +241,92 @@ __global__ void __launch_bounds__(256) trsm_kernel(float* A, int64_t n, int64_t 
     }
 }
 
-// C[M, N] += alpha * A[M, K] * op(B), K <= 64.  op(B) = B [K, N] row-major, or
-// (BT) B^T with B stored [N, K] row-major.  128 x 128 tiles, 256 threads, 8 x 8
-// outputs per thread from K-major shared tiles.  LOWER skips tiles that lie
-// entirely above the diagonal (n0 > m0 + 127).
-template <bool BT, bool LOWER>
-__global__ void __launch_bounds__(256) gemm_k64_kernel(float* C, int64_t ldc, const float* A, int64_t lda,
-                                                       const float* B, int64_t ldb, int64_t M, int64_t N, int K,
-                                                       float alpha) {
+// C[M, N] += alpha * op(A) * op(B).  op(A) = A [M, K] row-major, or (AT) A^T
+// with A stored [K, M] row-major; op(B) = B [K, N] row-major, or (BT) B^T with
+// B stored [N, K] row-major.  128 x 128 tiles, 256 threads, 8 x 8 outputs per
+// thread, K in stages of 32 through two shared buffers filled by cp.async
+// (global to shared without registers) while the other stage is multiplied.
+// LOWER skips tiles entirely above the diagonal (n0 > m0 + 127).  VEC: C rows
+// and the column base are 16-byte aligned, so the epilogue moves float4s.
+constexpr int kBK = 32;
+
+__device__ __forceinline__ void cp_async4(float* dst, const float* src, bool valid) {
+    const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
+    const int n = valid ? 4 : 0;                    // 0: zero-fill, nothing is read
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(d), "l"(src), "r"(n) : "memory");
+}
+
+template <bool AT, bool BT, bool LOWER, bool VEC>
+__global__ void __launch_bounds__(256, 2) gemm_kernel(float* C, int64_t ldc, const float* A, int64_t lda,
+                                                      const float* B, int64_t ldb, int64_t M, int64_t N, int K,
+                                                      float alpha) {
     extern __shared__ __align__(16) float smem[];
-    float* As = smem;                 // [64][kLd]: As[k][m]
-    float* Bs = smem + kP * kLd;      // [64][kLd]: Bs[k][n]
+    float* As = smem;                         // [2][kBK][kLd]: As[b][k][m]
+    float* Bs = smem + 2 * kBK * kLd;         // [2][kBK][kLd]: Bs[b][k][n]
     const int64_t m0 = (int64_t)blockIdx.y * 128, n0 = (int64_t)blockIdx.x * 128;
     if (LOWER && n0 > m0 + 127) return;
-    for (int e = threadIdx.x; e < 128 * kP; e += 256) {
-        const int mm = e / kP, k = e % kP;
-        As[k * kLd + mm] = (k < K && m0 + mm < M) ? A[(m0 + mm) * lda + k] : 0.0f;
-    }
-    if (BT) {
-        for (int e = threadIdx.x; e < 128 * kP; e += 256) {
-            const int nn = e / kP, k = e % kP;
-            Bs[k * kLd + nn] = (k < K && n0 + nn < N) ? B[(n0 + nn) * ldb + k] : 0.0f;
+    const int tid = threadIdx.x;
+    // element e = tid + 256*i of a 128 x 32 (A) or 32 x 128 (B) stage tile
+    auto issue = [&](int k0, int b) {
+        float* as = As + b * kBK * kLd;
+        float* bs = Bs + b * kBK * kLd;
+#pragma unroll
+        for (int i = 0; i < 16; i++) {
+            const int e = tid + 256 * i;
+            if (AT) {
+                const int k = e / 128, mm = e % 128;
+                const bool ok = k0 + k < K && m0 + mm < M;
+                cp_async4(as + k * kLd + mm, ok ? A + (int64_t)(k0 + k) * lda + m0 + mm : A, ok);
+            } else {
+                const int mm = e / kBK, k = e % kBK;
+                const bool ok = k0 + k < K && m0 + mm < M;
+                cp_async4(as + k * kLd + mm, ok ? A + (m0 + mm) * lda + k0 + k : A, ok);
+            }
+            if (BT) {
+                const int nn = e / kBK, k = e % kBK;
+                const bool ok = k0 + k < K && n0 + nn < N;
+                cp_async4(bs + k * kLd + nn, ok ? B + (n0 + nn) * ldb + k0 + k : B, ok);
+            } else {
+                const int k = e / 128, nn = e % 128;
+                const bool ok = k0 + k < K && n0 + nn < N;
+                cp_async4(bs + k * kLd + nn, ok ? B + (int64_t)(k0 + k) * ldb + n0 + nn : B, ok);
+            }
         }
-    } else {
-        for (int e = threadIdx.x; e < 128 * kP; e += 256) {
-            const int k = e / 128, nn = e % 128;
-            Bs[k * kLd + nn] = (k < K && n0 + nn < N) ? B[k * ldb + n0 + nn] : 0.0f;
-        }
-    }
-    __syncthreads();
-    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    const int tx = tid & 15, ty = tid >> 4;
     float acc[8][8];
 #pragma unroll
     for (int i = 0; i < 8; i++)
 #pragma unroll
         for (int j = 0; j < 8; j++) acc[i][j] = 0.0f;
-#pragma unroll 4
-    for (int k = 0; k < K; k++) {
-        const float4 a0 = *reinterpret_cast<const float4*>(As + k * kLd + ty * 4);
-        const float4 a1 = *reinterpret_cast<const float4*>(As + k * kLd + 64 + ty * 4);
-        const float4 b0 = *reinterpret_cast<const float4*>(Bs + k * kLd + tx * 4);
-        const float4 b1 = *reinterpret_cast<const float4*>(Bs + k * kLd + 64 + tx * 4);
-        const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-        const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+    const int nst = (K + kBK - 1) / kBK;
+    issue(0, 0);
+    for (int st = 0; st < nst; st++) {
+        const int b = st & 1;
+        if (st + 1 < nst) {
+            issue((st + 1) * kBK, b ^ 1);
+            asm volatile("cp.async.wait_group 1;" ::: "memory");
+        } else {
+            asm volatile("cp.async.wait_group 0;" ::: "memory");
+        }
+        __syncthreads();
+        const float* as = As + b * kBK * kLd;
+        const float* bs = Bs + b * kBK * kLd;
+#pragma unroll 8
+        for (int k = 0; k < kBK; k++) {
+            const float4 a0 = *reinterpret_cast<const float4*>(as + k * kLd + ty * 4);
+            const float4 a1 = *reinterpret_cast<const float4*>(as + k * kLd + 64 + ty * 4);
+            const float4 b0 = *reinterpret_cast<const float4*>(bs + k * kLd + tx * 4);
+            const float4 b1 = *reinterpret_cast<const float4*>(bs + k * kLd + 64 + tx * 4);
+            const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+            const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
-        for (int i = 0; i < 8; i++)
+            for (int i = 0; i < 8; i++)
 #pragma unroll
-            for (int j = 0; j < 8; j++) acc[i][j] = __fmaf_rn(av[i], bv[j], acc[i][j]);
+                for (int j = 0; j < 8; j++) acc[i][j] = __fmaf_rn(av[i], bv[j], acc[i][j]);
+        }
+        __syncthreads();                           // buffer b is refilled by the next issue
     }
 #pragma unroll
     for (int i = 0; i < 8; i++) {
@@ -236,30 +334,49 @@ __global__ void __launch_bounds__(256) gemm_k64_kernel(float* C, int64_t ldc, co
         if (r >= M) continue;
         float* crow = C + r * ldc;
 #pragma unroll
-        for (int j = 0; j < 8; j++) {
-            const int64_t c = n0 + (j < 4 ? tx * 4 + j : 64 + tx * 4 + j - 4);
-            if (c < N) crow[c] = __fmaf_rn(alpha, acc[i][j], crow[c]);
+        for (int h = 0; h < 2; h++) {
+            const int64_t c = n0 + h * 64 + tx * 4;
+            if (VEC && c + 3 < N) {
+                float4 v = *reinterpret_cast<float4*>(crow + c);
+                v.x = __fmaf_rn(alpha, acc[i][4 * h + 0], v.x);
+                v.y = __fmaf_rn(alpha, acc[i][4 * h + 1], v.y);
+                v.z = __fmaf_rn(alpha, acc[i][4 * h + 2], v.z);
+                v.w = __fmaf_rn(alpha, acc[i][4 * h + 3], v.w);
+                *reinterpret_cast<float4*>(crow + c) = v;
+            } else {
+#pragma unroll
+                for (int j = 0; j < 4; j++)
+                    if (c + j < N) crow[c + j] = __fmaf_rn(alpha, acc[i][4 * h + j], crow[c + j]);
+            }
         }
     }
 }
 
-template <bool BT, bool LOWER>
-cudaError_t launch_gemm(float* C, int64_t ldc, const float* A, int64_t lda, const float* B, int64_t ldb, int64_t M,
-                        int64_t N, int K, float alpha, cudaStream_t s) {
-    if (M <= 0 || N <= 0 || K <= 0) return cudaSuccess;
-    constexpr int kSmem = 2 * kP * kLd * (int)sizeof(float);
+template <bool AT, bool BT, bool LOWER, bool VEC>
+cudaError_t launch_gemm_t(float* C, int64_t ldc, const float* A, int64_t lda, const float* B, int64_t ldb, int64_t M,
+                          int64_t N, int K, float alpha, cudaStream_t s) {
+    constexpr int kSmem = 4 * kBK * kLd * (int)sizeof(float);
     static bool attr_set[64] = {false};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64 || !attr_set[dev]) {
-        e = cudaFuncSetAttribute(gemm_k64_kernel<BT, LOWER>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+        e = cudaFuncSetAttribute(gemm_kernel<AT, BT, LOWER, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
         if (e != cudaSuccess) return e;
         if (dev >= 0 && dev < 64) attr_set[dev] = true;
     }
     const dim3 grid((unsigned)((N + 127) / 128), (unsigned)((M + 127) / 128));
-    gemm_k64_kernel<BT, LOWER><<<grid, 256, kSmem, s>>>(C, ldc, A, lda, B, ldb, M, N, K, alpha);
+    gemm_kernel<AT, BT, LOWER, VEC><<<grid, 256, kSmem, s>>>(C, ldc, A, lda, B, ldb, M, N, K, alpha);
     return cudaGetLastError();
+}
+
+template <bool AT, bool BT, bool LOWER>
+cudaError_t launch_gemm(float* C, int64_t ldc, const float* A, int64_t lda, const float* B, int64_t ldb, int64_t M,
+                        int64_t N, int K, float alpha, cudaStream_t s) {
+    if (M <= 0 || N <= 0 || K <= 0) return cudaSuccess;
+    const bool vec = (ldc % 4 == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
+    return vec ? launch_gemm_t<AT, BT, LOWER, true>(C, ldc, A, lda, B, ldb, M, N, K, alpha, s)
+               : launch_gemm_t<AT, BT, LOWER, false>(C, ldc, A, lda, B, ldb, M, N, K, alpha, s);
 }
 
 __global__ void diag_d_kernel(const float* A, int64_t n, float* D) {
@@ -309,55 +426,78 @@ __device__ __forceinline__ float load_w(const void* W, int64_t idx) {
     return static_cast<const float*>(W)[idx];
 }
 
-// T[r][k] = W[r][perm[k]]
+// T[r][k] = Wp[r][k] = W[r][perm[k]] (fp32) and sfp[r][k] = sf[r][perm[k] / block].
 template <int DT>
-__global__ void __launch_bounds__(256) gather_w_kernel(const void* W, int64_t rows, int64_t n, const int32_t* perm,
-                                                       float* T, int* status) {
-    for (int64_t r = blockIdx.x; r < rows; r += gridDim.x)
-        for (int64_t k = threadIdx.x; k < n; k += blockDim.x)
-            T[r * n + k] = load_w<DT>(W, r * n + checked_index(perm[k], n, status));
+__global__ void __launch_bounds__(256) gather_w_kernel(LdlqParams p) {
+    for (int64_t r = blockIdx.x; r < p.rows; r += gridDim.x)
+        for (int64_t k = threadIdx.x; k < p.n; k += blockDim.x) {
+            const int64_t c = checked_index(p.perm[k], p.n, p.status);
+            const float v = load_w<DT>(p.W, r * p.n + c);
+            p.T[r * p.n + k] = v;
+            p.Wp[r * p.n + k] = v;
+            uint8_t code = p.sf[r * p.kb + c / p.block];
+            p.sfp[r * p.n + k] = code > 126 ? 0 : code;      // 0x7F (NaN) and above: a zero scale
+        }
 }
 
+// One LDLQ panel of P <= 64 columns (P % 16 == 0), one thread per row: the
+// row's 64 targets live in registers, column s is quantized at its fixed scale,
+// its error goes to EpT[s][r] and is fed to the later columns of the panel
+// through up[s][j] = U[k0+s][k0+j] (j > s).  The CTA's 128 rows of original
+// weights and scale codes for the panel are staged in shared memory with
+// coalesced loads first, so the sequential column walk reads only shared
+// memory.  The nibbles are written as one 64-byte run per row.
+constexpr int kPanelRows = 128;
+constexpr int kPanelSmem = (kP * kP + 128 + kPanelRows * (kP + 1)) * 4 + kPanelRows * (kP + 4);
+
 template <int DT>
-__global__ void __launch_bounds__(256) panel_kernel(LdlqParams p, int64_t k0, int P) {
-    __shared__ float up[kP][kP + 1];                 // up[s][j] = U[k0+s][k0+j] for s < j < P
+__global__ void __launch_bounds__(kPanelRows) panel_kernel(LdlqParams p, int64_t k0, int P, float* EpT) {
+    extern __shared__ __align__(16) float dsm[];
+    float (*up)[kP] = reinterpret_cast<float (*)[kP]>(dsm);                    // [kP][kP]
+    float* rtab = dsm + kP * kP;                                               // [128]
+    float (*wsm)[kP + 1] = reinterpret_cast<float (*)[kP + 1]>(rtab + 128);    // [kPanelRows][kP + 1]
+    uint8_t (*csm)[kP + 4] = reinterpret_cast<uint8_t (*)[kP + 4]>(wsm + kPanelRows);
     for (int e = threadIdx.x; e < kP * kP; e += blockDim.x) {
         const int s = e / kP, j = e % kP;
         up[s][j] = (s < j && j < P) ? p.U[(k0 + s) * p.n + k0 + j] : 0.0f;
     }
-    __syncthreads();
+    for (int c = threadIdx.x; c < 128; c += blockDim.x)
+        rtab[c] = (c >= 1 && c <= 126) ? __frcp_rn(f16bits_to_f32(e4m3_to_f16bits((uint32_t)c))) : 0.0f;
     const float S = __ldg(p.S);
     const float Einv = __frcp_rn(S);
     const bool usable = (S > 0.0f) && isfinite(S) && isfinite(Einv);
     const float E = usable ? Einv : 1.0f;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int64_t r = (int64_t)blockIdx.x * 8 + warp; r < p.rows; r += (int64_t)gridDim.x * 8) {
-        float t[2], w[2], v[2], rc[2];
-        int code[2];
-#pragma unroll
-        for (int h = 0; h < 2; h++) {
-            const int j = lane + 32 * h;
-            t[h] = w[h] = v[h] = rc[h] = 0.0f;
-            code[h] = 0;
-            if (j < P) {
-                const int64_t c = checked_index(p.perm[k0 + j], p.n, p.status);
-                t[h] = p.T[r * p.n + k0 + j];
-                w[h] = load_w<DT>(p.W, r * p.n + c);
-                code[h] = p.sf[r * p.kb + c / p.block];
-                if (code[h] > 126) code[h] = 0;              // 0x7F (NaN) and above: treated as a zero scale
-                v[h] = f16bits_to_f32(e4m3_to_f16bits((uint32_t)code[h]));
-                rc[h] = code[h] ? __frcp_rn(v[h]) : 0.0f;
-            }
+    for (int64_t rb = (int64_t)blockIdx.x * kPanelRows; rb < p.rows; rb += (int64_t)gridDim.x * kPanelRows) {
+        __syncthreads();                              // previous row block done with wsm/csm
+        for (int e = threadIdx.x; e < kPanelRows * kP; e += blockDim.x) {
+            const int rr = e / kP, j = e % kP;
+            const bool ok = rb + rr < p.rows && j < P;
+            wsm[rr][j] = ok ? p.Wp[(rb + rr) * p.n + k0 + j] : 0.0f;
+            csm[rr][j] = ok ? p.sfp[(rb + rr) * p.n + k0 + j] : 0;
         }
-        for (int s = 0; s < P; s++) {
-            const int owner = s & 31;
-            const bool hi = s >= 32;
-            float e = 0.0f;
-            if (lane == owner) {
-                const float ts = hi ? t[1] : t[0], ws = hi ? w[1] : w[0];
-                const float vs = hi ? v[1] : v[0], rs = hi ? rc[1] : rc[0];
-                const int cs = hi ? code[1] : code[0];
-                const float y = usable ? __fmul_rn(ts, E) : ts;
+        __syncthreads();
+        const int64_t r = rb + threadIdx.x;
+        if (r >= p.rows) continue;
+        const float* trow = p.T + r * p.n + k0;
+        const float* wrow = wsm[threadIdx.x];
+        const uint8_t* crow = csm[threadIdx.x];
+        float t[kP];
+#pragma unroll
+        for (int g = 0; g < kP / 4; g++) {
+            const float4 v = 4 * g < P ? *reinterpret_cast<const float4*>(trow + 4 * g) : make_float4(0, 0, 0, 0);
+            t[4 * g] = v.x;
+            t[4 * g + 1] = v.y;
+            t[4 * g + 2] = v.z;
+            t[4 * g + 3] = v.w;
+        }
+        uint32_t packed[kP / 4];
+#pragma unroll
+        for (int g = 0; g < kP / 4; g++) packed[g] = 0;
+#pragma unroll
+        for (int s = 0; s < kP; s++) {
+            if (s < P) {
+                const int cs = crow[s];
+                const float y = usable ? __fmul_rn(t[s], E) : t[s];
                 uint32_t nib;
                 float val;
                 if (y == 0.0f) {
@@ -367,22 +507,32 @@ __global__ void __launch_bounds__(256) panel_kernel(LdlqParams p, int64_t k0, in
                     nib = signbit(y) ? 8u : 0u;
                     val = signbit(y) ? -0.0f : 0.0f;
                 } else {
-                    const float tq = __fmul_rn(y, rs);
+                    const float tq = __fmul_rn(y, rtab[cs]);
                     nib = e2m1x2(tq, 0.0f) & 0xFu;
                     uint32_t h2;
                     asm("{\n\t.reg .b8 b;\n\tcvt.u8.u32 b, %1;\n\tcvt.rn.f16x2.e2m1x2 %0, b;\n\t}"
                         : "=r"(h2) : "r"(nib));
                     const float q = f16bits_to_f32((uint16_t)(h2 & 0xFFFFu));
-                    val = __fmul_rn(__fmul_rn(q, vs), S);
+                    const float v = f16bits_to_f32(e4m3_to_f16bits((uint32_t)cs));
+                    val = __fmul_rn(__fmul_rn(q, v), S);
                 }
-                e = __fsub_rn(ws, val);
-                p.qb[r * p.n + k0 + s] = (uint8_t)nib;
-                p.Ep[r * kP + s] = e;
+                const float e = __fsub_rn(wrow[s], val);
+                packed[s / 4] |= nib << (8 * (s % 4));
+                EpT[(int64_t)s * p.rows + r] = e;
+#pragma unroll
+                for (int g = (s + 1) / 4; g < kP / 4; g++) {
+                    const float4 u = *reinterpret_cast<const float4*>(&up[s][4 * g]);
+                    if (4 * g + 0 > s) t[4 * g + 0] = __fmaf_rn(e, u.x, t[4 * g + 0]);
+                    if (4 * g + 1 > s) t[4 * g + 1] = __fmaf_rn(e, u.y, t[4 * g + 1]);
+                    if (4 * g + 2 > s) t[4 * g + 2] = __fmaf_rn(e, u.z, t[4 * g + 2]);
+                    if (4 * g + 3 > s) t[4 * g + 3] = __fmaf_rn(e, u.w, t[4 * g + 3]);
+                }
             }
-            e = __shfl_sync(0xffffffffu, e, owner);
-            t[0] = __fmaf_rn(e, up[s][lane], t[0]);
-            t[1] = __fmaf_rn(e, up[s][lane + 32], t[1]);
         }
+        uint4* qrow = reinterpret_cast<uint4*>(p.qb + r * p.n + k0);
+#pragma unroll
+        for (int g = 0; g < kP / 16; g++)
+            if (16 * g < P) qrow[g] = make_uint4(packed[4 * g], packed[4 * g + 1], packed[4 * g + 2], packed[4 * g + 3]);
     }
 }
 
@@ -425,7 +575,7 @@ cudaError_t launch_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* 
             const unsigned tg = (unsigned)imin64((rest + 7) / 8, (int64_t)sms * 8);
             trsm_kernel<<<tg, 256, 0, s>>>(U, n, k0, nb, Linv);
             float* P = U + (k0 + nb) * n + k0;
-            e = launch_gemm<true, true>(U + (k0 + nb) * n + k0 + nb, n, P, n, P, n, rest, rest, nb, -1.0f, s);
+            e = launch_gemm<false, true, true>(U + (k0 + nb) * n + k0 + nb, n, P, n, P, n, rest, rest, nb, -1.0f, s);
             if (e != cudaSuccess) return e;
         }
         e = cudaGetLastError();
@@ -437,42 +587,71 @@ cudaError_t launch_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* 
     return cudaGetLastError();
 }
 
+// Workspace: T and Wp [rows, n] f32, qb and sfp [rows, n] bytes, EpT [kLdlqPanel, rows] f32, inv [n].
 size_t ldlq_quantize_workspace(int64_t rows, int64_t n) {
     auto up = [](int64_t b) { return (b + 255) / 256 * 256; };
-    return (size_t)(up(rows * n * 4) + up(rows * n) + up(rows * kP * 4) + up(n * 4));
+    return (size_t)(2 * up(rows * n * 4) + 2 * up(rows * n) + up((int64_t)kLdlqPanel * rows * 4) + up(n * 4));
 }
 
+// Columns in super-panels of kLdlqPanel (256): each 64-column panel is walked by
+// panel_kernel and its errors update the rest of the super-panel at once (K = 64);
+// after the super-panel, one GEMM with K = 256 updates every later column, so the
+// targets are read and written once per 256 columns.
 cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* ws, int sms, cudaStream_t s) {
     if (p.rows <= 0 || p.n <= 0) return cudaSuccess;
     auto up = [](int64_t b) { return (b + 255) / 256 * 256; };
     char* w = static_cast<char*>(ws);
+    const int64_t mat4 = up(p.rows * p.n * 4), mat1 = up(p.rows * p.n);
     p.T = reinterpret_cast<float*>(w);
-    p.qb = reinterpret_cast<uint8_t*>(w + up(p.rows * p.n * 4));
-    p.Ep = reinterpret_cast<float*>(w + up(p.rows * p.n * 4) + up(p.rows * p.n));
-    int32_t* inv = reinterpret_cast<int32_t*>(w + up(p.rows * p.n * 4) + up(p.rows * p.n) + up(p.rows * kP * 4));
+    p.Wp = reinterpret_cast<float*>(w + mat4);
+    p.qb = reinterpret_cast<uint8_t*>(w + 2 * mat4);
+    p.sfp = reinterpret_cast<uint8_t*>(w + 2 * mat4 + mat1);
+    float* EpT = reinterpret_cast<float*>(w + 2 * mat4 + 2 * mat1);
+    int32_t* inv = reinterpret_cast<int32_t*>(w + 2 * mat4 + 2 * mat1 + up((int64_t)kLdlqPanel * p.rows * 4));
     cudaError_t e = cudaMemsetAsync(inv, 0, (size_t)p.n * 4, s);
     if (e != cudaSuccess) return e;
     invperm_kernel<<<(unsigned)((p.n + 255) / 256), 256, 0, s>>>(p.perm, p.n, inv, p.status);
     const unsigned rg = (unsigned)imin64(p.rows, (int64_t)sms * 8);
     if (dtype == 0)
-        gather_w_kernel<0><<<rg, 256, 0, s>>>(p.W, p.rows, p.n, p.perm, p.T, p.status);
+        gather_w_kernel<0><<<rg, 256, 0, s>>>(p);
     else
-        gather_w_kernel<1><<<rg, 256, 0, s>>>(p.W, p.rows, p.n, p.perm, p.T, p.status);
+        gather_w_kernel<1><<<rg, 256, 0, s>>>(p);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    const unsigned pg = (unsigned)imin64((p.rows + 7) / 8, (int64_t)sms * 4);
-    for (int64_t k0 = 0; k0 < p.n; k0 += kP) {
-        const int P = (int)imin64(kP, p.n - k0);
-        if (dtype == 0)
-            panel_kernel<0><<<pg, 256, 0, s>>>(p, k0, P);
-        else
-            panel_kernel<1><<<pg, 256, 0, s>>>(p, k0, P);
-        e = cudaGetLastError();
+    static bool attr_set[64] = {false};
+    int dev = 0;
+    e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64 || !attr_set[dev]) {
+        e = cudaFuncSetAttribute(panel_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPanelSmem);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(panel_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPanelSmem);
         if (e != cudaSuccess) return e;
-        const int64_t rest = p.n - k0 - P;
+        if (dev >= 0 && dev < 64) attr_set[dev] = true;
+    }
+    const unsigned pg = (unsigned)imin64((p.rows + kPanelRows - 1) / kPanelRows, (int64_t)sms * 8);
+    for (int64_t s0 = 0; s0 < p.n; s0 += kLdlqPanel) {
+        const int64_t span = imin64(kLdlqPanel, p.n - s0);
+        for (int64_t k0 = s0; k0 < s0 + span; k0 += kP) {
+            const int P = (int)imin64(kP, s0 + span - k0);
+            float* Ek = EpT + (k0 - s0) * p.rows;
+            if (dtype == 0)
+                panel_kernel<0><<<pg, kPanelRows, kPanelSmem, s>>>(p, k0, P, Ek);
+            else
+                panel_kernel<1><<<pg, kPanelRows, kPanelSmem, s>>>(p, k0, P, Ek);
+            e = cudaGetLastError();
+            if (e != cudaSuccess) return e;
+            const int64_t rest_in = s0 + span - (k0 + P);
+            if (rest_in > 0) {
+                e = launch_gemm<true, false, false>(p.T + k0 + P, p.n, Ek, p.rows, p.U + k0 * p.n + k0 + P, p.n,
+                                                    p.rows, rest_in, P, 1.0f, s);
+                if (e != cudaSuccess) return e;
+            }
+        }
+        const int64_t rest = p.n - (s0 + span);
         if (rest > 0) {
-            e = launch_gemm<false, false>(p.T + k0 + P, p.n, p.Ep, kP, p.U + k0 * p.n + k0 + P, p.n, p.rows, rest, P,
-                                          1.0f, s);
+            e = launch_gemm<true, false, false>(p.T + s0 + span, p.n, EpT, p.rows, p.U + s0 * p.n + s0 + span, p.n,
+                                                p.rows, rest, (int)span, 1.0f, s);
             if (e != cudaSuccess) return e;
         }
     }
