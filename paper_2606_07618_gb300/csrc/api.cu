@@ -9,6 +9,7 @@
 
 #include <cuda_runtime.h>
 
+#include "ldlq_kernels.h"
 #include "nvfp4_kernels.h"
 #include "nvfp4ss.h"
 

@@ -23,6 +23,7 @@
 #include <cuda_bf16.h>
 
 #include "nvfp4_device.cuh"
+#include "ldlq_kernels.h"
 #include "nvfp4_kernels.h"
 
 namespace nvfp4 {
