@@ -2,6 +2,7 @@
 // overlap checks (all before any launch), then dispatch to the kernels.  The
 // library never allocates, frees or synchronises; every call is asynchronous on
 // the caller's stream.
+#include <atomic>
 #include <climits>
 #include <cmath>
 #include <cstdint>
@@ -18,13 +19,16 @@ using namespace nvfp4;
 namespace {
 
 int sm_count() {
-    static int cache[64] = {0};
+    static std::atomic<int> cache[64];           // zero-initialised; 0 = not looked up yet
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 0;
-    if (dev < 64 && cache[dev] > 0) return cache[dev];
+    if (dev < 64) {
+        const int c = cache[dev].load(std::memory_order_relaxed);
+        if (c > 0) return c;
+    }
     int n = 0;
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    if (dev < 64) cache[dev] = n;
+    if (dev < 64) cache[dev].store(n, std::memory_order_relaxed);
     return n;
 }
 

@@ -20,6 +20,8 @@
 // Q follows the sweep's float32 contract: y = fl(t*E), q = RNE_E2M1(fl(y*r_c)),
 // What = fl(fl(q*v_c)*S); a zero-scale block or an unusable S gives signed
 // zeros; an exactly zero y takes the +0 code.
+#include <atomic>
+
 #include <cuda_bf16.h>
 
 #include "nvfp4_device.cuh"
@@ -357,14 +359,14 @@ template <bool AT, bool BT, bool LOWER, bool VEC>
 cudaError_t launch_gemm_t(float* C, int64_t ldc, const float* A, int64_t lda, const float* B, int64_t ldb, int64_t M,
                           int64_t N, int K, float alpha, cudaStream_t s) {
     constexpr int kSmem = 4 * kBK * kLd * (int)sizeof(float);
-    static bool attr_set[64] = {false};
+    static std::atomic<bool> attr_set[64];        // per device: the shared-memory opt-in is done
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 64 || !attr_set[dev]) {
+    if (dev < 0 || dev >= 64 || !attr_set[dev].load(std::memory_order_acquire)) {
         e = cudaFuncSetAttribute(gemm_kernel<AT, BT, LOWER, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
         if (e != cudaSuccess) return e;
-        if (dev >= 0 && dev < 64) attr_set[dev] = true;
+        if (dev >= 0 && dev < 64) attr_set[dev].store(true, std::memory_order_release);
     }
     const dim3 grid((unsigned)((N + 127) / 128), (unsigned)((M + 127) / 128));
     gemm_kernel<AT, BT, LOWER, VEC><<<grid, 256, kSmem, s>>>(C, ldc, A, lda, B, ldb, M, N, K, alpha);
@@ -619,16 +621,16 @@ cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* 
         gather_w_kernel<1><<<rg, 256, 0, s>>>(p);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    static bool attr_set[64] = {false};
+    static std::atomic<bool> attr_set[64];        // per device: the shared-memory opt-in is done
     int dev = 0;
     e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 64 || !attr_set[dev]) {
+    if (dev < 0 || dev >= 64 || !attr_set[dev].load(std::memory_order_acquire)) {
         e = cudaFuncSetAttribute(panel_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPanelSmem);
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(panel_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPanelSmem);
         if (e != cudaSuccess) return e;
-        if (dev >= 0 && dev < 64) attr_set[dev] = true;
+        if (dev >= 0 && dev < 64) attr_set[dev].store(true, std::memory_order_release);
     }
     const unsigned pg = (unsigned)imin64((p.rows + kPanelRows - 1) / kPanelRows, (int64_t)sms * 8);
     for (int64_t s0 = 0; s0 < p.n; s0 += kLdlqPanel) {
