@@ -443,26 +443,28 @@ __global__ void __launch_bounds__(256) gather_w_kernel(LdlqParams p) {
         }
 }
 
-// One LDLQ panel of P <= 64 columns (P % 16 == 0), one thread per row: the
-// row's 64 targets live in registers, column s is quantized at its fixed scale,
-// its error goes to EpT[s][r] and is fed to the later columns of the panel
-// through up[s][j] = U[k0+s][k0+j] (j > s).  The CTA's 128 rows of original
-// weights and scale codes for the panel are staged in shared memory with
-// coalesced loads first, so the sequential column walk reads only shared
-// memory.  The nibbles are written as one 64-byte run per row.
-constexpr int kPanelRows = 128;
+// One LDLQ panel of P <= 64 columns (P % 16 == 0).  Four threads per row
+// (adjacent lanes), thread k of a row owning columns 16k..16k+15 in registers:
+// at column s the owner quantizes it at its fixed scale, writes the error to
+// EpT[s][r], and the error reaches the other three threads by shuffle; each
+// thread then updates its 16 targets through up[s][c] = U[k0+s][k0+c] (zero for
+// c <= s and past the panel).  Splitting the 64-wide update shortens the
+// sequential chain per column four-fold.  The CTA's 32 rows of original weights
+// and scale codes are staged in shared memory with coalesced loads first.
+constexpr int kPanelThreads = 128;
+constexpr int kPanelRows = kPanelThreads / 4;
 constexpr int kPanelSmem = (kP * kP + 128 + kPanelRows * (kP + 1)) * 4 + kPanelRows * (kP + 4);
 
 template <int DT>
-__global__ void __launch_bounds__(kPanelRows) panel_kernel(LdlqParams p, int64_t k0, int P, float* EpT) {
+__global__ void __launch_bounds__(kPanelThreads) panel_kernel(LdlqParams p, int64_t k0, int P, float* EpT) {
     extern __shared__ __align__(16) float dsm[];
     float (*up)[kP] = reinterpret_cast<float (*)[kP]>(dsm);                    // [kP][kP]
     float* rtab = dsm + kP * kP;                                               // [128]
     float (*wsm)[kP + 1] = reinterpret_cast<float (*)[kP + 1]>(rtab + 128);    // [kPanelRows][kP + 1]
     uint8_t (*csm)[kP + 4] = reinterpret_cast<uint8_t (*)[kP + 4]>(wsm + kPanelRows);
     for (int e = threadIdx.x; e < kP * kP; e += blockDim.x) {
-        const int s = e / kP, j = e % kP;
-        up[s][j] = (s < j && j < P) ? p.U[(k0 + s) * p.n + k0 + j] : 0.0f;
+        const int s = e / kP, c = e % kP;
+        up[s][c] = (s < c && c < P) ? p.U[(k0 + s) * p.n + k0 + c] : 0.0f;
     }
     for (int c = threadIdx.x; c < 128; c += blockDim.x)
         rtab[c] = (c >= 1 && c <= 126) ? __frcp_rn(f16bits_to_f32(e4m3_to_f16bits((uint32_t)c))) : 0.0f;
@@ -470,72 +472,93 @@ __global__ void __launch_bounds__(kPanelRows) panel_kernel(LdlqParams p, int64_t
     const float Einv = __frcp_rn(S);
     const bool usable = (S > 0.0f) && isfinite(S) && isfinite(Einv);
     const float E = usable ? Einv : 1.0f;
+    const int lane = threadIdx.x & 31;
+    const int kq = threadIdx.x & 3;                   // this thread's quarter of the columns
+    const int rr = threadIdx.x >> 2;                  // row within the CTA's block
     for (int64_t rb = (int64_t)blockIdx.x * kPanelRows; rb < p.rows; rb += (int64_t)gridDim.x * kPanelRows) {
         __syncthreads();                              // previous row block done with wsm/csm
-        for (int e = threadIdx.x; e < kPanelRows * kP; e += blockDim.x) {
-            const int rr = e / kP, j = e % kP;
-            const bool ok = rb + rr < p.rows && j < P;
-            wsm[rr][j] = ok ? p.Wp[(rb + rr) * p.n + k0 + j] : 0.0f;
-            csm[rr][j] = ok ? p.sfp[(rb + rr) * p.n + k0 + j] : 0;
+        {
+            float4 wv[kPanelRows * kP / 4 / kPanelThreads];
+            uint32_t cv[kPanelRows * kP / 4 / kPanelThreads];
+#pragma unroll
+            for (int u = 0; u < kPanelRows * kP / 4 / kPanelThreads; u++) {
+                const int e = threadIdx.x + kPanelThreads * u, row = e / (kP / 4), j = 4 * (e % (kP / 4));
+                const bool ok = rb + row < p.rows && j < P;
+                wv[u] = ok ? *reinterpret_cast<const float4*>(p.Wp + (rb + row) * p.n + k0 + j) : make_float4(0, 0, 0, 0);
+                cv[u] = ok ? *reinterpret_cast<const uint32_t*>(p.sfp + (rb + row) * p.n + k0 + j) : 0u;
+            }
+#pragma unroll
+            for (int u = 0; u < kPanelRows * kP / 4 / kPanelThreads; u++) {
+                const int e = threadIdx.x + kPanelThreads * u, row = e / (kP / 4), j = 4 * (e % (kP / 4));
+                wsm[row][j] = wv[u].x;
+                wsm[row][j + 1] = wv[u].y;
+                wsm[row][j + 2] = wv[u].z;
+                wsm[row][j + 3] = wv[u].w;
+                *reinterpret_cast<uint32_t*>(&csm[row][j]) = cv[u];
+            }
         }
         __syncthreads();
-        const int64_t r = rb + threadIdx.x;
-        if (r >= p.rows) continue;
-        const float* trow = p.T + r * p.n + k0;
-        const float* wrow = wsm[threadIdx.x];
-        const uint8_t* crow = csm[threadIdx.x];
-        float t[kP];
+        const int64_t r = rb + rr;
+        const bool active = r < p.rows;               // a whole quad shares r
+        const int c0 = 16 * kq;
+        float t[16];
 #pragma unroll
-        for (int g = 0; g < kP / 4; g++) {
-            const float4 v = 4 * g < P ? *reinterpret_cast<const float4*>(trow + 4 * g) : make_float4(0, 0, 0, 0);
+        for (int g = 0; g < 4; g++) {
+            const float4 v = (active && c0 + 4 * g < P) ? *reinterpret_cast<const float4*>(p.T + r * p.n + k0 + c0 + 4 * g)
+                                                        : make_float4(0, 0, 0, 0);
             t[4 * g] = v.x;
             t[4 * g + 1] = v.y;
             t[4 * g + 2] = v.z;
             t[4 * g + 3] = v.w;
         }
-        uint32_t packed[kP / 4];
+        uint32_t packed[4] = {0, 0, 0, 0};
+#pragma unroll 1
+        for (int kb = 0; kb < P / 16; kb++) {          // the quarter whose columns are walked now
+            const bool owner = kq == kb;
+            const int src = (lane & ~3) | kb;
 #pragma unroll
-        for (int g = 0; g < kP / 4; g++) packed[g] = 0;
-#pragma unroll
-        for (int s = 0; s < kP; s++) {
-            if (s < P) {
-                const int cs = crow[s];
-                const float y = usable ? __fmul_rn(t[s], E) : t[s];
-                uint32_t nib;
-                float val;
-                if (y == 0.0f) {
-                    nib = 0;
-                    val = 0.0f;
-                } else if (!usable || cs == 0) {
-                    nib = signbit(y) ? 8u : 0u;
-                    val = signbit(y) ? -0.0f : 0.0f;
-                } else {
-                    const float tq = __fmul_rn(y, rtab[cs]);
-                    nib = e2m1x2(tq, 0.0f) & 0xFu;
-                    uint32_t h2;
-                    asm("{\n\t.reg .b8 b;\n\tcvt.u8.u32 b, %1;\n\tcvt.rn.f16x2.e2m1x2 %0, b;\n\t}"
-                        : "=r"(h2) : "r"(nib));
-                    const float q = f16bits_to_f32((uint16_t)(h2 & 0xFFFFu));
-                    const float v = f16bits_to_f32(e4m3_to_f16bits((uint32_t)cs));
-                    val = __fmul_rn(__fmul_rn(q, v), S);
+            for (int j = 0; j < 16; j++) {
+                const int s = 16 * kb + j;
+                float e = 0.0f;
+                if (owner && active) {
+                    const int cs = csm[rr][s];
+                    const float y = usable ? __fmul_rn(t[j], E) : t[j];
+                    uint32_t nib;
+                    float val;
+                    if (y == 0.0f) {
+                        nib = 0;
+                        val = 0.0f;
+                    } else if (!usable || cs == 0) {
+                        nib = signbit(y) ? 8u : 0u;
+                        val = signbit(y) ? -0.0f : 0.0f;
+                    } else {
+                        const float tq = __fmul_rn(y, rtab[cs]);
+                        nib = e2m1x2(tq, 0.0f) & 0xFu;
+                        uint32_t h2;
+                        asm("{\n\t.reg .b8 b;\n\tcvt.u8.u32 b, %1;\n\tcvt.rn.f16x2.e2m1x2 %0, b;\n\t}"
+                            : "=r"(h2) : "r"(nib));
+                        const float qv = f16bits_to_f32((uint16_t)(h2 & 0xFFFFu));
+                        const float v = f16bits_to_f32(e4m3_to_f16bits((uint32_t)cs));
+                        val = __fmul_rn(__fmul_rn(qv, v), S);
+                    }
+                    e = __fsub_rn(wsm[rr][s], val);
+                    packed[j / 4] |= nib << (8 * (j % 4));
+                    EpT[(int64_t)s * p.rows + r] = e;
                 }
-                const float e = __fsub_rn(wrow[s], val);
-                packed[s / 4] |= nib << (8 * (s % 4));
-                EpT[(int64_t)s * p.rows + r] = e;
+                e = __shfl_sync(0xffffffffu, e, src);
+                const float* us = &up[s][c0];
 #pragma unroll
-                for (int g = (s + 1) / 4; g < kP / 4; g++) {
-                    const float4 u = *reinterpret_cast<const float4*>(&up[s][4 * g]);
-                    if (4 * g + 0 > s) t[4 * g + 0] = __fmaf_rn(e, u.x, t[4 * g + 0]);
-                    if (4 * g + 1 > s) t[4 * g + 1] = __fmaf_rn(e, u.y, t[4 * g + 1]);
-                    if (4 * g + 2 > s) t[4 * g + 2] = __fmaf_rn(e, u.z, t[4 * g + 2]);
-                    if (4 * g + 3 > s) t[4 * g + 3] = __fmaf_rn(e, u.w, t[4 * g + 3]);
+                for (int g = 0; g < 4; g++) {
+                    const float4 u = *reinterpret_cast<const float4*>(us + 4 * g);
+                    t[4 * g + 0] = __fmaf_rn(e, u.x, t[4 * g + 0]);
+                    t[4 * g + 1] = __fmaf_rn(e, u.y, t[4 * g + 1]);
+                    t[4 * g + 2] = __fmaf_rn(e, u.z, t[4 * g + 2]);
+                    t[4 * g + 3] = __fmaf_rn(e, u.w, t[4 * g + 3]);
                 }
             }
         }
-        uint4* qrow = reinterpret_cast<uint4*>(p.qb + r * p.n + k0);
-#pragma unroll
-        for (int g = 0; g < kP / 16; g++)
-            if (16 * g < P) qrow[g] = make_uint4(packed[4 * g], packed[4 * g + 1], packed[4 * g + 2], packed[4 * g + 3]);
+        if (active && c0 < P)
+            *reinterpret_cast<uint4*>(p.qb + r * p.n + k0 + c0) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
     }
 }
 
@@ -632,16 +655,16 @@ cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* 
         if (e != cudaSuccess) return e;
         if (dev >= 0 && dev < 64) attr_set[dev].store(true, std::memory_order_release);
     }
-    const unsigned pg = (unsigned)imin64((p.rows + kPanelRows - 1) / kPanelRows, (int64_t)sms * 8);
+    const unsigned pg = (unsigned)imin64((p.rows + kPanelRows - 1) / kPanelRows, (int64_t)sms * 16);
     for (int64_t s0 = 0; s0 < p.n; s0 += kLdlqPanel) {
         const int64_t span = imin64(kLdlqPanel, p.n - s0);
         for (int64_t k0 = s0; k0 < s0 + span; k0 += kP) {
             const int P = (int)imin64(kP, s0 + span - k0);
             float* Ek = EpT + (k0 - s0) * p.rows;
             if (dtype == 0)
-                panel_kernel<0><<<pg, kPanelRows, kPanelSmem, s>>>(p, k0, P, Ek);
+                panel_kernel<0><<<pg, kPanelThreads, kPanelSmem, s>>>(p, k0, P, Ek);
             else
-                panel_kernel<1><<<pg, kPanelRows, kPanelSmem, s>>>(p, k0, P, Ek);
+                panel_kernel<1><<<pg, kPanelThreads, kPanelSmem, s>>>(p, k0, P, Ek);
             e = cudaGetLastError();
             if (e != cudaSuccess) return e;
             const int64_t rest_in = s0 + span - (k0 + P);
