@@ -133,12 +133,11 @@ def make_inputs(device: str):
     return wl, xs, ws
 
 
-def sweep_traffic_per_launch(elems_per_launch):
-    """DRAM bytes per sweep launch from the committed ncu capture
-    (profiles/quantize_kernel_wmse_traffic.json), scaled by elements; None if
-    the kernel sources changed since the capture."""
+def traffic_per_launch(record, elems_per_launch):
+    """DRAM bytes per launch from a committed ncu capture (profiles/<record>),
+    scaled by elements; None if the kernel sources changed since the capture."""
     import hashlib
-    path = os.path.join(ROOT, "profiles", "quantize_kernel_wmse_traffic.json")
+    path = os.path.join(ROOT, "profiles", record)
     try:
         with open(path) as f:
             rec = json.load(f)
@@ -195,13 +194,25 @@ def run_gpu(args, rank, world):
         B.scalesweep_quantize(xs[i], 16, S[i:i + 1], B.NVFP4_OBJ_WMSE, ws[i], 0, *win, o["codes"], o["sf_linear"],
                               o["sf_swizzled"], None, stream=stream)
 
+    # The step: one grouped launch over the 7 tensors that also reduces every
+    # tensor's global scale (a ninth warp per CTA streams the reductions while
+    # the other eight sweep).  The same step as per-tensor launches is timed as
+    # a leg: global scales on a side stream, sweep i after amax i.
     aux = torch.cuda.Stream()
     wsps = [torch.empty_like(wsp) for _ in xs]
     amax_done = [torch.cuda.Event() for _ in xs]
+    gws = torch.empty(B.scalesweep_quantize_group_workspace(), dtype=torch.uint8, device=dev)
+    desc = B.group_descriptors(xs, ws, [0] * len(xs), [o["codes"] for o in outs], [o["sf_linear"] for o in outs],
+                               [o["sf_swizzled"] for o in outs])
 
     def step(events=None):
-        # The global scales run on a side stream: amax(i+1) (HBM-bound) overlaps
-        # sweep(i) (ALU-bound); sweep(i) waits only for amax(i).
+        if events is not None:
+            events[0].record(stream)
+        B.scalesweep_quantize_group(desc, B.NVFP4_IN_BF16, B.NVFP4_OBJ_WMSE, D, S, st, gws, stream=stream)
+        if events is not None:
+            events[1].record(stream)
+
+    def step_per_tensor():
         aux.wait_stream(stream)
         with torch.cuda.stream(aux):
             for i, x in enumerate(xs):
@@ -209,14 +220,10 @@ def run_gpu(args, rank, world):
                 amax_done[i].record(aux)
         for i in range(len(xs)):
             stream.wait_event(amax_done[i])
-            if events is not None:
-                events[i][0].record(stream)
             sweep(i)
-            if events is not None:
-                events[i][1].record(stream)
         stream.wait_stream(aux)
 
-    launches_per_step = 3 * len(xs)   # amax partial + final + sweep per tensor (shapes need no pad kernel)
+    launches_per_step = 1   # the grouped kernel (the workspace reset is a memset; these shapes need no pad kernel)
 
     for _ in range(args.warmup):
         step()
@@ -224,7 +231,7 @@ def run_gpu(args, rank, world):
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in xs] for _ in range(args.steps)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(torch.cuda.current_device()) as clk:
         t0.record(stream)
@@ -235,7 +242,7 @@ def run_gpu(args, rank, world):
     if world > 1:
         torch.distributed.barrier()
     ms = t0.elapsed_time(t1)
-    sweep_ms = sum(ev[k][i][0].elapsed_time(ev[k][i][1]) for k in range(args.steps) for i in range(len(xs)))
+    sweep_ms = sum(ev[k][0].elapsed_time(ev[k][1]) for k in range(args.steps))
     ms = reduce_max_ms(ms, world, dev)
     ms_step = ms / args.steps
     value = world * total / (ms_step * 1e-3) / 1e9
@@ -243,9 +250,12 @@ def run_gpu(args, rank, world):
     # status word: any non-finite input would have been flagged
     assert int(st.item()) == 0, "non-finite input detected"
 
-    # ---- roofline of the dominant kernel (sweep), from the events above
-    bpe = alg_bytes_per_elem()
-    alg_bytes = sum(n * bpe + 4 * x.shape[1] for n, x in zip(n_el, xs))     # + per-channel weights
+    # ---- roofline of the dominant (only) kernel, the grouped launch, from the events above
+    # algorithmic bytes: the global-scale reduction reads each input once, the
+    # sweep reads it again and writes codes and both scale layouts; plus the
+    # channel weights
+    bpe = alg_bytes_per_elem() + 2
+    alg_bytes = sum(n * bpe + 4 * x.shape[1] for n, x in zip(n_el, xs))
     sweep_s_per_step = sweep_ms / args.steps * 1e-3
     gbs = alg_bytes / sweep_s_per_step / 1e9
     hbm_peak, peak_kind = peaks()
@@ -260,12 +270,13 @@ def run_gpu(args, rank, world):
     alu_achieved = ops / sweep_s_per_step
     roofline = {"bound": "alu", "achieved": round(alu_achieved / 1e12, 3), "peak": round(alu_peak / 1e12, 3),
                 "unit": "Tops/s", "frac": round(alu_achieved / alu_peak, 4), "traffic": None,
-                "kernel": "quantize_kernel<bf16,ScaleSweep,WMSE,16>",
+                "kernel": "quantize_group_kernel<bf16,WMSE,dynamic S> (7 tensors, one launch per step)",
                 "peak_note": f"{nsm} SMs x 128 FP32 lanes x median SM clock {sm_mhz} MHz",
                 "hbm": {"achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s", "frac": round(gbs / hbm_peak, 4),
                         "peak_kind": peak_kind, "bytes_per_elem": bpe},
-                "sweep_ms_per_step": round(sweep_s_per_step * 1e3, 4)}
-    roofline["traffic"] = sweep_traffic_per_launch(total / len(xs))
+                "launch_ms": round(sweep_s_per_step * 1e3, 4),
+                "launch_note": "events around the call: the 256-byte workspace memset and the kernel"}
+    roofline["traffic"] = traffic_per_launch("quantize_group_kernel_wmse_traffic.json", total)
 
     # ---- overhead vs the AbsMax kernel on the same tensors, same S and layouts
     def time_leg(fn, reps):
@@ -313,7 +324,12 @@ def run_gpu(args, rank, world):
         for i, x in enumerate(xs):
             B.nvfp4_global_scale(x, D, S[i:i + 1], st, wsp, stream=stream)
 
+    def sweep_group_static():
+        B.scalesweep_quantize_group(desc, B.NVFP4_IN_BF16, B.NVFP4_OBJ_WMSE, 0.0, S, st, None, stream=stream)
+
     reps = max(3, min(50, args.steps))
+    t_pt = time_leg(step_per_tensor, reps)
+    t_gs = time_leg(sweep_group_static, reps)
     t_abs = time_leg(absmax_all, reps)
     t_ss = time_leg(sweep_all, reps)
     t_ssm = time_leg(sweep_mse_all, reps)
@@ -321,7 +337,9 @@ def run_gpu(args, rank, world):
     t_dq = time_leg(dequant_all, reps)
     t_am = time_leg(amax_all, reps)
     gel = lambda ms_: round(total / (ms_ * 1e-3) / 1e9, 2)
-    legs = {"scalesweep_wmse": {"ms": round(t_ss, 4), "gelem_s": gel(t_ss)},
+    legs = {"step_per_tensor_launches": {"ms": round(t_pt, 4), "gelem_s": gel(t_pt)},
+            "scalesweep_wmse_grouped_static_scales": {"ms": round(t_gs, 4), "gelem_s": gel(t_gs)},
+            "scalesweep_wmse": {"ms": round(t_ss, 4), "gelem_s": gel(t_ss)},
             "scalesweep_mse": {"ms": round(t_ssm, 4), "gelem_s": gel(t_ssm)},
             "absmax": {"ms": round(t_abs, 4), "gelem_s": gel(t_abs)},
             "four_over_six_wmse": {"ms": round(t_46, 4), "gelem_s": gel(t_46)},
@@ -496,7 +514,9 @@ def config_dict(wl, world):
             "elements": wl.numel, "input": "bf16", "block": wl.block, "objective": wl.objective,
             "global_scale": f"amax/(6*{int(wl.fp8_div)}) computed every step", "scale_layouts": "linear+swizzled",
             "parallelism": f"replicas{world}" if world > 1 else "single-gpu",
-            "l2": "no flush: each step streams 436 MB of inputs (> 129 MB L2); the amax passes run on a side stream, sweep i waits for amax i only"}
+            "l2": "no flush: each step streams the 436 MB of inputs (> 129 MB L2) twice, once for the global scales "
+                  "and once for the sweep; inside the one launch tensor i+1's scale is reduced while tensor i is "
+                  "swept"}
 
 
 def run_kernel_case(args):
@@ -533,6 +553,33 @@ def run_kernel_case(args):
         "wmse_fused": lambda: B.scalesweep_quantize_dynamic(x, args.block, 256.0, 1, w, 0, *win, S, None, dws,
                                                             o["codes"], o["sf_linear"], o["sf_swizzled"]),
     }
+    S1 = torch.empty(1, device=dev)
+    gws = torch.empty(B.scalesweep_quantize_group_workspace(), dtype=torch.uint8, device=dev)
+    d1 = B.group_descriptors([x], [w], [0], [o["codes"]], [o["sf_linear"]], [o["sf_swizzled"]])
+    fns["sweep_wmse_group"] = lambda: B.scalesweep_quantize_group(d1, B.NVFP4_IN_BF16, 1, 0.0, S, None, None)
+    fns["wmse_group_dynamic"] = lambda: B.scalesweep_quantize_group(d1, B.NVFP4_IN_BF16, 1, 256.0, S1, None, gws)
+    if args.kernel_case.startswith(("group_layer", "layer_")):
+        # the Llama-3-8B layer in one grouped launch (dynamic scales), as the bench step
+        _, xs, wl_ws = make_inputs(dev)
+        lo = [B.empty_outputs(t.shape[0], t.shape[1], 16, device=dev, linear=True, swizzled=True) for t in xs]
+        dl = B.group_descriptors(xs, wl_ws, [0] * len(xs), [q["codes"] for q in lo], [q["sf_linear"] for q in lo],
+                                 [q["sf_swizzled"] for q in lo])
+        SL = torch.empty(len(xs), device=dev)
+        fns["group_layer"] = lambda: B.scalesweep_quantize_group(dl, B.NVFP4_IN_BF16, 1, 256.0, SL, None, gws)
+        SS = torch.empty(len(xs), device=dev)
+        B.scalesweep_quantize_group(dl, B.NVFP4_IN_BF16, 1, 256.0, SS, None, gws)
+        fns["group_layer_static"] = lambda: B.scalesweep_quantize_group(dl, B.NVFP4_IN_BF16, 1, 0.0, SS, None, None)
+        dlin = B.group_descriptors(xs, wl_ws, [0] * len(xs), [q["codes"] for q in lo], [q["sf_linear"] for q in lo],
+                                   [None] * len(xs))
+        fns["group_layer_linear"] = lambda: B.scalesweep_quantize_group(dlin, B.NVFP4_IN_BF16, 1, 256.0, SL, None, gws)
+        fns["group_layer_static_linear"] = lambda: B.scalesweep_quantize_group(dlin, B.NVFP4_IN_BF16, 1, 0.0, SS, None,
+                                                                               None)
+        fns["layer_per_tensor_static"] = lambda: [
+            B.scalesweep_quantize(t, 16, SS[i:i + 1], 1, wl_ws[i], 0, *win, lo[i]["codes"], lo[i]["sf_linear"],
+                                  lo[i]["sf_swizzled"]) for i, t in enumerate(xs)]
+        n = sum(t.numel() for t in xs)
+    else:
+        n = x.numel()
     fn = fns[args.kernel_case]
     fns["sweep_mse"]()
     for _ in range(2):
@@ -545,7 +592,6 @@ def run_kernel_case(args):
     b.record()
     torch.cuda.synchronize()
     ms = a.elapsed_time(b) / args.reps
-    n = x.numel()
     print(json.dumps({"kernel_case": args.kernel_case, "rows": args.rows, "cols": args.cols, "block": args.block,
                       "ms": round(ms, 4), "gelem_s": round(n / ms / 1e6, 2)}), flush=True)
 
@@ -796,6 +842,8 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=64)
     ap.add_argument("--kernel-case", default=None,
                     choices=["sweep_wmse", "sweep_mse", "absmax", "four_six", "dequant", "amax", "mse_two_launch",
+                             "sweep_wmse_group", "wmse_group_dynamic", "group_layer", "group_layer_static",
+                             "layer_per_tensor_static", "group_layer_linear", "group_layer_static_linear",
                              "mse_fused", "wmse_fused"])
     ap.add_argument("--rows", type=int, default=16384)
     ap.add_argument("--cols", type=int, default=8192)

@@ -165,6 +165,62 @@ nvfp4_status scalesweep_quantize_dynamic(const void* x, nvfp4_dtype dt, int64_t 
                                          float* block_loss, void* stream);
 
 /*
+ * One tensor of a grouped call (scalesweep_quantize_group).  Fields as the
+ * arguments of scalesweep_quantize with block = 16:
+ *   x             [rows, cols] of the call's dtype, 16-byte aligned, cols % 16 == 0.
+ *   w             WMSE importance (w[row*w_row_stride + col], 16-byte aligned;
+ *                 w_row_stride 0 broadcasts one [cols] vector); NULL for MSE.
+ *   codes         [rows, cols/2], 8-byte aligned.
+ *   sf_linear     optional [rows, cols/16]; sf_swizzled optional 128x4-atom
+ *                 layout; at least one of the two.
+ */
+typedef struct {
+    const void* x;
+    int64_t rows, cols;
+    const float* w;
+    int64_t w_row_stride;
+    uint8_t* codes;
+    uint8_t* sf_linear;
+    uint8_t* sf_swizzled;
+} nvfp4_group_tensor;
+
+#define NVFP4_GROUP_MAX 16
+
+/*
+ * Bytes of device workspace scalesweep_quantize_group needs.
+ */
+size_t scalesweep_quantize_group_workspace(void);
+
+/*
+ * ScaleSweep quantisation of `count` tensors (1..NVFP4_GROUP_MAX, e.g. all
+ * linear weights of one transformer layer) in one launch: for every tensor the
+ * result of scalesweep_quantize with block 16 and the default window ([-3, 7]
+ * MSE, [-8, 7] WMSE, Sec. 4.2.2), bit for bit.  The segments of all tensors are
+ * walked by one grid, so the call has a single launch tail instead of one per
+ * tensor.
+ *   tensors     host array of `count` descriptors, read during the call only.
+ *   dt, obj     input type and objective, shared by all tensors.
+ *   fp8_div     0: static global scales, S[i] is read for tensor i.
+ *               > 0: per-call (dynamic) global scales, S[i] = fl32(amax_i /
+ *               fl32(6*fp8_div)) over tensor i (Sec. 4.2.1) is computed in the
+ *               same launch and written; tensor i's reduction overlaps the sweep
+ *               of the smaller tensors before it (cooperative launch, preceded
+ *               by a cudaMemsetAsync of the workspace counters).
+ *   S           device float[count].
+ *   status_dev  optional device int: bit 0 OR-ed in for NaN/inf input (dynamic
+ *               only), bit 1 if a wait for a scale timed out (about a second per
+ *               wait; outputs are then incomplete -- a resident grid makes this
+ *               unreachable in practice).
+ *   workspace   scalesweep_quantize_group_workspace() bytes, 16-byte aligned, no
+ *               initialisation (dynamic only; may be NULL for static scales).
+ * Outputs must not overlap any input, S, status_dev, the workspace or each
+ * other.  Concurrent calls must use distinct workspaces.
+ */
+nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt,
+                                       nvfp4_objective obj, float fp8_div, float* S, int* status_dev,
+                                       void* workspace, size_t ws_bytes, void* stream);
+
+/*
  * AbsMax quantisation with the global scale computed in the same launch, as
  * scalesweep_quantize_dynamic (baseline for the fused dynamic path).
  */

@@ -32,6 +32,15 @@ class Nvfp4Error(RuntimeError):
 
 _lib = None
 
+NVFP4_GROUP_MAX = 16
+
+
+class GroupTensor(ctypes.Structure):
+    """nvfp4_group_tensor: one tensor of a scalesweep_quantize_group call."""
+    _fields_ = [("x", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64), ("w", ctypes.c_void_p),
+                ("w_row_stride", ctypes.c_int64), ("codes", ctypes.c_void_p), ("sf_linear", ctypes.c_void_p),
+                ("sf_swizzled", ctypes.c_void_p)]
+
 
 def library_path() -> str:
     return _build.LIB
@@ -58,6 +67,8 @@ def lib() -> ctypes.CDLL:
         L.nvfp4_dynamic_workspace.argtypes, L.nvfp4_dynamic_workspace.restype = [], sz
         L.scalesweep_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, i, p, i64, i, i, p, p, p, sz, p, p, p, p, p]
         L.absmax_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, p, p, p, sz, p, p, p, p, p]
+        L.scalesweep_quantize_group_workspace.argtypes, L.scalesweep_quantize_group_workspace.restype = [], sz
+        L.scalesweep_quantize_group.argtypes = [ctypes.POINTER(GroupTensor), i, i, i, f, p, p, p, sz, p]
         L.nvfp4_optimal_scale.argtypes = [p, i, i64, i64, i, p, i, p, i64, p, p, p, p, p]
         L.nvfp4_ldlq_prepare_workspace.argtypes, L.nvfp4_ldlq_prepare_workspace.restype = [i64], sz
         L.nvfp4_ldlq_prepare.argtypes = [p, i64, f, p, p, p, p, p, sz, p]
@@ -65,7 +76,8 @@ def lib() -> ctypes.CDLL:
         L.ldlq_quantize.argtypes = [p, i, i64, i64, i, p, p, p, p, p, p, p, sz, p]
         for fn in ("nvfp4_global_scale", "nvfp4_global_scale_noalloc", "scalesweep_quantize", "absmax_quantize",
                    "four_over_six_quantize", "nvfp4_dequantize", "scalesweep_quantize_dynamic",
-                   "absmax_quantize_dynamic", "nvfp4_optimal_scale", "nvfp4_ldlq_prepare", "ldlq_quantize"):
+                   "absmax_quantize_dynamic", "nvfp4_optimal_scale", "nvfp4_ldlq_prepare", "ldlq_quantize",
+                   "scalesweep_quantize_group"):
             getattr(L, fn).restype = i
         _lib = L
     return _lib
@@ -172,6 +184,35 @@ def absmax_quantize_dynamic(x, block: int, fp8_div: float, S_out, status, worksp
                                        _ptr(status), _ptr(workspace), ws_bytes, _ptr(codes), _ptr(sf_linear),
                                        _ptr(sf_swizzled), _ptr(block_loss), _stream(stream))
     _check("absmax_quantize_dynamic", rc)
+
+
+def scalesweep_quantize_group_workspace() -> int:
+    return int(lib().scalesweep_quantize_group_workspace())
+
+
+def group_descriptors(xs, ws, w_row_strides, codes, sf_linear, sf_swizzled):
+    """The nvfp4_group_tensor array for tensors xs[i] with weights ws[i] (None
+    for MSE) and output buffers codes[i], sf_linear[i], sf_swizzled[i] (None
+    where not wanted).  Reusable across calls on the same buffers."""
+    n = len(xs)
+    arr = (GroupTensor * n)()
+    for i, x in enumerate(xs):
+        rows, cols = x.shape
+        arr[i] = GroupTensor(x.data_ptr(), rows, cols, ws[i].data_ptr() if ws[i] is not None else None,
+                             int(w_row_strides[i]), codes[i].data_ptr(),
+                             sf_linear[i].data_ptr() if sf_linear[i] is not None else None,
+                             sf_swizzled[i].data_ptr() if sf_swizzled[i] is not None else None)
+    return arr
+
+
+def scalesweep_quantize_group(desc, dtype: int, objective: int, fp8_div: float, S, status=None, workspace=None,
+                              stream=None):
+    """desc: the array from group_descriptors.  fp8_div 0 reads S[i]; > 0
+    computes and writes S[i] in the launch."""
+    ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    rc = lib().scalesweep_quantize_group(desc, len(desc), int(dtype), int(objective), float(fp8_div), _ptr(S),
+                                         _ptr(status), _ptr(workspace), ws_bytes, _stream(stream))
+    _check("scalesweep_quantize_group", rc)
 
 
 def nvfp4_optimal_scale(x, block: int, S, objective: int, w, w_row_stride: int, s_opt, loss_opt, fp8_code=None,

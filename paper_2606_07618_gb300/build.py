@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libnvfp4ss.so")
 SOURCES = ["api.cu", "quantize.cu", "quantize_dynamic.cu", "scale_dequant.cu", "global_scale_noalloc.cu",
-           "optimal_scale.cu", "ldlq.cu"]
+           "optimal_scale.cu", "ldlq.cu", "quantize_group.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -10,6 +10,7 @@
 
 #include <cuda_runtime.h>
 
+#include "group_kernels.h"
 #include "ldlq_kernels.h"
 #include "nvfp4_kernels.h"
 #include "nvfp4ss.h"
@@ -261,6 +262,128 @@ nvfp4_status scalesweep_quantize_dynamic(const void* x, nvfp4_dtype dt, int64_t 
     const DynArgs d{fp8_div, S_out, status_dev, workspace, ws_bytes};
     return quantize_common(0, x, dt, rows, cols, block, nullptr, obj, w, w_row_stride, win_lo, win_hi, codes,
                            sf_linear, sf_swizzled, block_loss, stream, &d);
+}
+
+static_assert(kGroupMax == NVFP4_GROUP_MAX, "group descriptor count");
+
+size_t scalesweep_quantize_group_workspace(void) { return kGroupWorkspace; }
+
+nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt,
+                                       nvfp4_objective obj, float fp8_div, float* S, int* status_dev,
+                                       void* workspace, size_t ws_bytes, void* stream) {
+    if (dt != NVFP4_IN_BF16 && dt != NVFP4_IN_F32) return NVFP4_ERR_INVALID_ARG;
+    if (obj != NVFP4_OBJ_MSE && obj != NVFP4_OBJ_WMSE) return NVFP4_ERR_INVALID_ARG;
+    if (!tensors || count < 1 || count > NVFP4_GROUP_MAX || !S) return NVFP4_ERR_INVALID_ARG;
+    const bool dyn = fp8_div != 0.0f;
+    if (dyn && (!(fp8_div > 0.0f) || fp8_div > 1e30f)) return NVFP4_ERR_INVALID_ARG;
+    if (dyn && (!workspace || ws_bytes < kGroupWorkspace)) return NVFP4_ERR_INVALID_ARG;
+    if (!aligned(S, 4) || (status_dev && !aligned(status_dev, 4)) || (workspace && !aligned(workspace, 16)))
+        return NVFP4_ERR_ALIGNMENT;
+    const int64_t esize = dt == NVFP4_IN_BF16 ? 2 : 4;
+
+    // Buffers the launch writes and reads, for the overlap checks.
+    constexpr int kMaxW = 3 * NVFP4_GROUP_MAX + 3, kMaxR = 2 * NVFP4_GROUP_MAX + 1;
+    const void* wp[kMaxW];
+    int64_t wl[kMaxW];
+    const void* rp[kMaxR];
+    int64_t rl[kMaxR];
+    int nw = 0, nr = 0;
+    auto add_w = [&](const void* q, int64_t n) { if (q && n > 0) { wp[nw] = q; wl[nw++] = n; } };
+    auto add_r = [&](const void* q, int64_t n) { if (q && n > 0) { rp[nr] = q; rl[nr++] = n; } };
+    if (dyn) add_w(S, 4 * (int64_t)count);
+    else add_r(S, 4 * (int64_t)count);
+    add_w(status_dev, 4);
+    if (dyn) add_w(workspace, (int64_t)ws_bytes);
+
+    Shape sh[NVFP4_GROUP_MAX];
+    for (int i = 0; i < count; i++) {
+        const nvfp4_group_tensor& t = tensors[i];
+        nvfp4_status st = check_shape(t.rows, t.cols, 16, &sh[i]);
+        if (st != NVFP4_OK) return st;
+        if (sh[i].n == 0) continue;
+        if (!t.x || !t.codes || (!t.sf_linear && !t.sf_swizzled)) return NVFP4_ERR_INVALID_ARG;
+        if (!aligned(t.x, 16) || !aligned(t.codes, 8)) return NVFP4_ERR_ALIGNMENT;
+        if (sh[i].n > INT64_MAX / 4) return NVFP4_ERR_RANGE;
+        int64_t wbytes = 0;
+        if (obj == NVFP4_OBJ_WMSE) {
+            if (!t.w || (t.w_row_stride != 0 && t.w_row_stride < t.cols)) return NVFP4_ERR_INVALID_ARG;
+            if (t.w_row_stride < 0 || t.w_row_stride % 4 != 0 || !aligned(t.w, 16)) return NVFP4_ERR_ALIGNMENT;
+            if (t.w_row_stride == 0) {
+                wbytes = t.cols * 4;
+            } else if (!mul_ok(t.rows - 1, t.w_row_stride, &wbytes) || wbytes > INT64_MAX / 4 - t.cols) {
+                return NVFP4_ERR_RANGE;
+            } else {
+                wbytes = (wbytes + t.cols) * 4;
+            }
+        }
+        add_r(t.x, sh[i].n * esize);
+        if (obj == NVFP4_OBJ_WMSE) add_r(t.w, wbytes);
+        add_w(t.codes, sh[i].n / 2);
+        add_w(t.sf_linear, sh[i].nblocks);
+        add_w(t.sf_swizzled, sh[i].sw_bytes);
+    }
+    for (int a = 0; a < nw; a++) {
+        for (int b = a + 1; b < nw; b++)
+            if (overlap(wp[a], wl[a], wp[b], wl[b])) return NVFP4_ERR_INVALID_ARG;
+        for (int b = 0; b < nr; b++)
+            if (overlap(wp[a], wl[a], rp[b], rl[b])) return NVFP4_ERR_INVALID_ARG;
+    }
+    for (int a = 0; a < nw; a++)
+        if (!device_accessible(wp[a])) return NVFP4_ERR_INVALID_ARG;
+    for (int b = 0; b < nr; b++)
+        if (!device_accessible(rp[b])) return NVFP4_ERR_INVALID_ARG;
+    if (!device_accessible(S)) return NVFP4_ERR_INVALID_ARG;
+    const int sms = sm_count();
+    if (sms <= 0) return NVFP4_ERR_CUDA;
+
+    // Processing order: ascending size (stable), so the reduction that cannot
+    // overlap a sweep (the first tensor's) is the smallest.
+    int order[NVFP4_GROUP_MAX];
+    for (int i = 0; i < count; i++) order[i] = i;
+    for (int i = 1; i < count; i++)
+        for (int k = i; k > 0 && sh[order[k]].n < sh[order[k - 1]].n; k--) {
+            const int tmp = order[k];
+            order[k] = order[k - 1];
+            order[k - 1] = tmp;
+        }
+    GroupParams p;
+    std::memset(&p, 0, sizeof(p));
+    int64_t rows[NVFP4_GROUP_MAX];
+    int64_t seg = 0;
+    for (int k = 0; k < count; k++) {
+        const int i = order[k];
+        const nvfp4_group_tensor& t = tensors[i];
+        GroupTensor& g = p.t[k];
+        g.x = t.x;
+        g.w = obj == NVFP4_OBJ_WMSE ? t.w : nullptr;
+        g.w_row_stride = t.w_row_stride;
+        g.codes = t.codes;
+        g.sf_linear = t.sf_linear;
+        g.sf_swizzled = t.sf_swizzled;
+        g.kb = sh[i].kb;
+        g.kpad4 = sh[i].kpad4;
+        g.nseg = sh[i].nseg;
+        g.seg_begin = seg;
+        g.nvec = sh[i].n * esize / 16;
+        g.narrow = sh[i].narrow;
+        if (g.narrow && g.kb > 0) g.kb_div = make_fast_div((uint32_t)g.kb);
+        g.s_index = i;
+        rows[k] = t.rows;
+        const int64_t unit = kGroupCtaSegments;          // a CTA's segments never straddle two tensors
+        if (g.nseg > INT64_MAX - seg - unit) return NVFP4_ERR_RANGE;
+        seg += (g.nseg + unit - 1) / unit * unit;
+    }
+    p.count = count;
+    p.dyn = dyn ? 1 : 0;
+    p.total_seg = seg;
+    p.fp8_div = fp8_div;
+    p.S = S;
+    p.status_dev = status_dev;
+    p.amax_bits = dyn ? static_cast<unsigned*>(workspace) : nullptr;
+    p.arrived = dyn ? static_cast<unsigned*>(workspace) + kGroupMax : nullptr;
+    const cudaError_t e = launch_quantize_group(p, rows, dt == NVFP4_IN_BF16 ? 0 : 1, obj == NVFP4_OBJ_WMSE ? 1 : 0,
+                                                sms, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
 }
 
 nvfp4_status absmax_quantize_dynamic(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,

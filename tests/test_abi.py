@@ -30,7 +30,7 @@ def test_header_declares_the_api():
         "scalesweep_quantize", "absmax_quantize", "four_over_six_quantize", "nvfp4_dequantize",
         "nvfp4_dynamic_workspace", "scalesweep_quantize_dynamic", "absmax_quantize_dynamic",
         "nvfp4_optimal_scale", "nvfp4_ldlq_prepare_workspace", "nvfp4_ldlq_prepare", "nvfp4_ldlq_workspace",
-        "ldlq_quantize"])
+        "ldlq_quantize", "scalesweep_quantize_group_workspace", "scalesweep_quantize_group"])
 
 
 def test_library_exports_every_declared_symbol(L):
@@ -113,3 +113,46 @@ def test_ldlq_validation_without_gpu(L):
     assert q(codes=FAKE) == 1                         # codes overlap W
     assert q(wsp=FAKE + 0x130000) == 1                # workspace overlaps U
 
+
+
+def test_group_validation_without_gpu(L):
+    """Argument checks of scalesweep_quantize_group that return before any CUDA
+    call (the overlap checks, which need device pointers to pass, are
+    exercised with real buffers in the GPU tests)."""
+    from paper_2606_07618_gb300 import binding as B
+    f = ctypes.c_float
+
+    def desc(first=None, every=None):
+        arr = (B.GroupTensor * 2)()
+        for i in range(2):
+            t = dict(x=FAKE + i * 0x100000, rows=4, cols=64, w=None, w_row_stride=0,
+                     codes=FAKE + 0x1000000 + i * 0x100000, sf_linear=FAKE + 0x2000000 + i * 0x100000,
+                     sf_swizzled=None)
+            t.update(every or {})
+            if i == 0:
+                t.update(first or {})
+            arr[i] = B.GroupTensor(**t)
+        return arr
+
+    S, st, ws = FAKE + 0x3000000, FAKE + 0x3000100, FAKE + 0x3001000
+    g = lambda d, n=2, dt=0, obj=0, div=256.0, S=S, ws=ws, wsb=256: \
+        L.scalesweep_quantize_group(d, n, dt, obj, f(div), S, st, ws, wsb, None)
+    assert L.scalesweep_quantize_group_workspace() >= 128
+    assert g(desc(), n=0) == 1                        # empty group
+    assert g(desc(), n=17) == 1                       # more than NVFP4_GROUP_MAX
+    assert g(desc(), dt=3) == 1
+    assert g(desc(), obj=2) == 1
+    assert g(desc(), div=-1.0) == 1
+    assert g(desc(), S=None) == 1
+    assert g(desc(), ws=None) == 1                    # dynamic scales need the workspace
+    assert g(desc(), wsb=16) == 1
+    assert g(desc(), ws=FAKE + 0x3001004) == 3
+    assert g(desc(), S=S + 2) == 3
+    assert g(desc({"cols": 40})) == 1                 # cols % 16
+    assert g(desc({"x": FAKE + 2})) == 3
+    assert g(desc({"codes": FAKE + 0x1000004})) == 3
+    assert g(desc({"sf_linear": None})) == 1          # no scale output
+    assert g(desc(), obj=1) == 1                      # WMSE needs weights
+    assert g(desc(every={"w": FAKE + 0x4000004}), obj=1) == 3
+    assert g(desc(every={"w": FAKE + 0x4000000, "w_row_stride": 8}), obj=1) == 1
+    assert g(desc({"rows": 2 ** 40, "cols": 2 ** 40})) == 4

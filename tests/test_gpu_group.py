@@ -1,0 +1,222 @@
+"""Grouped ScaleSweep launch (scalesweep_quantize_group) on the GPU.
+
+One launch quantises a list of tensors and, with a dynamic global scale,
+reduces each tensor's amax inside the same launch.  For every tensor it must
+give the oracle's codes and scales (near-tie rule of parity.py) and, bit for
+bit, what the per-tensor entry points give: nvfp4_global_scale then
+scalesweep_quantize (S, codes, linear and swizzled scales).  Shapes are
+ragged on purpose: segment counts that are not multiples of 32 (a warp), rows
+not multiples of 128 and scale columns not multiples of 4 (swizzle pads), a
+one-row tensor, an empty tensor, an all-zero tensor.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from parity import compare_quantize
+from paper_2606_07618_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+WIN = None
+
+
+@pytest.fixture(scope="module")
+def B():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_07618_gb300 import binding
+    binding.lib()
+    oracle.build()
+    global WIN
+    WIN = (binding.NVFP4_WINDOW_DEFAULT, binding.NVFP4_WINDOW_DEFAULT)
+    return binding
+
+
+SHAPES = [(130, 192), (1, 64), (37, 48), (300, 512), (0, 64), (2048, 1024), (64, 80)]
+
+
+def make_group(dtype, obj, seed=0, shapes=SHAPES, row_weights=(3,)):
+    xs, ws, strides = [], [], []
+    for i, (r, c) in enumerate(shapes):
+        if r == 0:
+            x = torch.empty(0, c, dtype=torch.bfloat16)
+        else:
+            x = W.small_tensor(r, c, 100 * seed + i, dist="student_t" if i % 2 else "normal", std=0.02 + 0.01 * i,
+                               outliers=1 + i % 3, mult=20.0 + i)
+        if i == 6 and r > 0:
+            x = torch.zeros(r, c, dtype=torch.bfloat16)          # an all-zero tensor: S = 0, signs only
+        xs.append(x.to(dtype))
+        if obj == 1:
+            g = torch.Generator().manual_seed(seed * 31 + i)
+            if i in row_weights:                                   # per-element weights, padded row stride
+                stride = c + 4
+                w = torch.exp(torch.randn(max(r, 1), stride, generator=g))
+            else:
+                stride = 0
+                w = torch.exp(torch.randn(c, generator=g))
+            ws.append(w)
+            strides.append(stride)
+        else:
+            ws.append(None)
+            strides.append(0)
+    return xs, ws, strides
+
+
+def run_group(B, xs, ws, strides, obj, D=256.0, S_in=None, ws_buf=None, status=None):
+    dev_x = [x.to(DEV) for x in xs]
+    dev_w = [w.to(DEV) if w is not None else None for w in ws]
+    outs = [B.empty_outputs(x.shape[0], x.shape[1], 16, device=DEV, linear=True, swizzled=True) for x in xs]
+    for o in outs:                                                   # poison: every byte must be written
+        o["codes"].fill_(0xEE)
+        o["sf_linear"].fill_(0xEE)
+        o["sf_swizzled"].fill_(0xEE)
+    desc = B.group_descriptors(dev_x, dev_w, strides, [o["codes"] for o in outs], [o["sf_linear"] for o in outs],
+                               [o["sf_swizzled"] for o in outs])
+    dt = B.NVFP4_IN_BF16 if xs[0].dtype == torch.bfloat16 else B.NVFP4_IN_F32
+    st = status if status is not None else torch.zeros(1, dtype=torch.int32, device=DEV)
+    if S_in is None:
+        S = torch.full((len(xs),), -1.0, device=DEV)
+        if ws_buf is None:
+            ws_buf = torch.empty(B.scalesweep_quantize_group_workspace(), dtype=torch.uint8, device=DEV)
+        B.scalesweep_quantize_group(desc, dt, obj, D, S, st, ws_buf)
+    else:
+        S = S_in.clone()
+        B.scalesweep_quantize_group(desc, dt, obj, 0.0, S, st, None)
+    torch.cuda.synchronize()
+    return S, st, outs, dev_x, dev_w
+
+
+def per_tensor(B, x, w, stride, obj, S=None, D=256.0):
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    if S is None:
+        S = torch.empty(1, device=DEV)
+        wsb = torch.empty(B.nvfp4_global_scale_workspace(x.numel()), dtype=torch.uint8, device=DEV)
+        B.nvfp4_global_scale(x, D, S, st, wsb)
+    o = B.empty_outputs(x.shape[0], x.shape[1], 16, device=DEV, linear=True, swizzled=True)
+    if x.numel():
+        B.scalesweep_quantize(x, 16, S, obj, w, stride, *WIN, o["codes"], o["sf_linear"], o["sf_swizzled"], None)
+    torch.cuda.synchronize()
+    return S, st, o
+
+
+def check_against_per_tensor(B, xs, ws, strides, obj, S, outs, dev_x, dev_w, static=False):
+    for i, x in enumerate(dev_x):
+        S1, _, o1 = per_tensor(B, x, dev_w[i], strides[i], obj, S=S[i:i + 1] if static else None)
+        if not static:
+            assert S[i].item() == S1.item(), f"tensor {i}: S {S[i].item()} vs {S1.item()}"
+        if x.numel() == 0:
+            continue
+        for k in ("codes", "sf_linear", "sf_swizzled"):
+            assert torch.equal(outs[i][k], o1[k]), f"tensor {i}: {k}"
+
+
+@pytest.mark.parametrize("obj", [0, 1])
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_group_dynamic_matches_oracle_and_per_tensor(B, dtype, obj):
+    xs, ws, strides = make_group(dtype, obj, seed=1)
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, obj)
+    assert st.item() == 0
+    check_against_per_tensor(B, xs, ws, strides, obj, S, outs, dev_x, dev_w)
+    for i, x in enumerate(xs):
+        xs_np = x.float().numpy()
+        So, bad = oracle.global_scale(xs_np, 256.0) if x.numel() else (0.0, False)
+        assert S[i].item() == np.float32(So), f"tensor {i}"
+        if x.numel() == 0:
+            continue
+        wn = ws[i].numpy() if ws[i] is not None else None
+        ref = oracle.quantize(0, xs_np, 16, So, obj, w=wn, w_row_stride=strides[i])
+        compare_quantize(xs_np, So, 16, obj, ws[i], strides[i], outs[i], ref)
+
+
+@pytest.mark.parametrize("obj", [0, 1])
+def test_group_static_scales(B, obj):
+    xs, ws, strides = make_group(torch.bfloat16, obj, seed=2)
+    S_in = torch.tensor([oracle.global_scale(x.float().numpy(), 448.0)[0] if x.numel() else 1.0 for x in xs],
+                        dtype=torch.float32, device=DEV)
+    S_in[2] = 0.0                                                  # a zero scale: signs only
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, obj, S_in=S_in)
+    assert torch.equal(S, S_in) and st.item() == 0
+    check_against_per_tensor(B, xs, ws, strides, obj, S, outs, dev_x, dev_w, static=True)
+
+
+def test_group_single_tensor_and_many_tensors(B):
+    # one tensor; and the maximum of 16 tensors of assorted small shapes
+    xs, ws, strides = make_group(torch.bfloat16, 1, seed=3, shapes=[(513, 4096)], row_weights=())
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, 1)
+    check_against_per_tensor(B, xs, ws, strides, 1, S, outs, dev_x, dev_w)
+    shapes = [(1 + 37 * i, 16 * (1 + (5 * i) % 23)) for i in range(16)]
+    xs, ws, strides = make_group(torch.bfloat16, 0, seed=4, shapes=shapes)
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, 0)
+    assert st.item() == 0
+    check_against_per_tensor(B, xs, ws, strides, 0, S, outs, dev_x, dev_w)
+
+
+def test_group_llama_layer_full_size(B):
+    """The Llama-3-8B layer (7 weights, 218M elements, WMSE with lognormal
+    channel weights, dynamic S, D = 256) in one launch: every tensor equals the
+    per-tensor path bit for bit; S and 24 sampled rows per tensor equal the
+    oracle."""
+    wl = W.workload("llama8b")
+    xs = [W.draw(t) for t in wl.tensors]
+    ws = [W.draw_weights(t) for t in wl.tensors]
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, [0] * len(xs), 1, D=wl.fp8_div)
+    assert st.item() == 0
+    check_against_per_tensor(B, xs, ws, [0] * len(xs), 1, S, outs, dev_x, dev_w)
+    for i, (t, x) in enumerate(zip(wl.tensors, xs)):
+        xs_np = x.float().numpy()
+        So, _ = oracle.global_scale(xs_np, wl.fp8_div)
+        assert S[i].item() == np.float32(So), t.name
+        idx = np.unique(np.linspace(0, t.rows - 1, 24).astype(np.int64))
+        sub = {"codes": outs[i]["codes"][idx], "sf_linear": outs[i]["sf_linear"][idx]}
+        ref = oracle.quantize(0, xs_np[idx], 16, So, 1, w=ws[i].numpy())
+        compare_quantize(xs_np[idx], So, 16, 1, ws[i], 0, sub, ref)
+
+
+def test_group_nonfinite_flag_reuse_and_empty(B):
+    xs, ws, strides = make_group(torch.bfloat16, 0, seed=5)
+    wsb = torch.empty(B.scalesweep_quantize_group_workspace(), dtype=torch.uint8, device=DEV)
+    ref = None
+    for _ in range(3):                                             # one workspace, back to back
+        S, st, outs, _, _ = run_group(B, xs, ws, strides, 0, ws_buf=wsb)
+        assert st.item() == 0
+        if ref is None:
+            ref = (S.clone(), outs)
+        else:
+            assert torch.equal(S, ref[0])
+            for a, b in zip(outs, ref[1]):
+                for k in ("codes", "sf_linear", "sf_swizzled"):
+                    assert torch.equal(a[k], b[k])
+    bad = [x.clone() for x in xs]
+    bad[3][5, 7] = float("inf")
+    S, st, _, _, _ = run_group(B, bad, ws, strides, 0, ws_buf=wsb)
+    assert st.item() & 1
+    assert S[3].item() == float("inf") and torch.equal(S[:3], ref[0][:3])
+    bad = [x.clone() for x in xs]
+    bad[5][0, 0] = float("nan")
+    S, st, _, _, _ = run_group(B, bad, ws, strides, 0, ws_buf=wsb)
+    assert st.item() & 1 and S[5].item() == ref[0][5].item()         # NaN is skipped by the max
+    empty = [torch.empty(0, 64, dtype=torch.bfloat16), torch.empty(3, 0, dtype=torch.bfloat16)]
+    S, st, _, _, _ = run_group(B, empty, [None, None], [0, 0], 0, ws_buf=wsb)
+    assert S.tolist() == [0.0, 0.0] and st.item() == 0
+
+
+def test_group_rejects_overlapping_buffers(B):
+    x = torch.zeros(64, 64, dtype=torch.bfloat16, device=DEV)
+    codes = torch.empty(64, 32, dtype=torch.uint8, device=DEV)
+    sf = torch.empty(64, 4, dtype=torch.uint8, device=DEV)
+    S = torch.zeros(2, device=DEV)
+    wsb = torch.empty(B.scalesweep_quantize_group_workspace(), dtype=torch.uint8, device=DEV)
+    both = B.group_descriptors([x, x], [None, None], [0, 0], [codes, codes], [sf, None], [None, sf])
+    with pytest.raises(B.Nvfp4Error) as e:
+        B.scalesweep_quantize_group(both, B.NVFP4_IN_BF16, 0, 256.0, S, None, wsb)
+    assert e.value.code == 1
+    into_input = B.group_descriptors([x], [None], [0], [x.view(torch.uint8)[:, :32]], [sf], [None])
+    with pytest.raises(B.Nvfp4Error) as e:
+        B.scalesweep_quantize_group(into_input, B.NVFP4_IN_BF16, 0, 256.0, S, None, wsb)
+    assert e.value.code == 1
+    ok = B.group_descriptors([x], [None], [0], [codes], [sf], [None])
+    B.scalesweep_quantize_group(ok, B.NVFP4_IN_BF16, 0, 256.0, S, None, wsb)
+    torch.cuda.synchronize()
+    assert S[0].item() == 0.0 and not torch.any(codes & 0x77).item()
