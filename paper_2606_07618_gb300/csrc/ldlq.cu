@@ -298,11 +298,14 @@ __global__ void __launch_bounds__(256, 2) gemm_kernel(float* C, int64_t ldc, con
         asm volatile("cp.async.commit_group;" ::: "memory");
     };
     const int tx = tid & 15, ty = tid >> 4;
-    float acc[8][8];
+    // 8 x 8 outputs per thread as 8 x 4 packed pairs: one fma.rn.f32x2 per pair
+    // (per lane the same IEEE fma as the scalar form, at twice the operands per
+    // register read).
+    u64 acc[8][4];
 #pragma unroll
     for (int i = 0; i < 8; i++)
 #pragma unroll
-        for (int j = 0; j < 8; j++) acc[i][j] = 0.0f;
+        for (int j = 0; j < 4; j++) acc[i][j] = 0ull;
     const int nst = (K + kBK - 1) / kBK;
     issue(0, 0);
     for (int st = 0; st < nst; st++) {
@@ -323,11 +326,13 @@ __global__ void __launch_bounds__(256, 2) gemm_kernel(float* C, int64_t ldc, con
             const float4 b0 = *reinterpret_cast<const float4*>(bs + k * kLd + tx * 4);
             const float4 b1 = *reinterpret_cast<const float4*>(bs + k * kLd + 64 + tx * 4);
             const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-            const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+            const u64 bp[4] = {pack2(b0.x, b0.y), pack2(b0.z, b0.w), pack2(b1.x, b1.y), pack2(b1.z, b1.w)};
 #pragma unroll
-            for (int i = 0; i < 8; i++)
+            for (int i = 0; i < 8; i++) {
+                const u64 ap = pack2(av[i], av[i]);
 #pragma unroll
-                for (int j = 0; j < 8; j++) acc[i][j] = __fmaf_rn(av[i], bv[j], acc[i][j]);
+                for (int j = 0; j < 4; j++) acc[i][j] = fma2(ap, bp[j], acc[i][j]);
+            }
         }
         __syncthreads();                           // buffer b is refilled by the next issue
     }
@@ -339,17 +344,20 @@ __global__ void __launch_bounds__(256, 2) gemm_kernel(float* C, int64_t ldc, con
 #pragma unroll
         for (int h = 0; h < 2; h++) {
             const int64_t c = n0 + h * 64 + tx * 4;
+            float o[4];
+            unpack2(acc[i][2 * h], o[0], o[1]);
+            unpack2(acc[i][2 * h + 1], o[2], o[3]);
             if (VEC && c + 3 < N) {
                 float4 v = *reinterpret_cast<float4*>(crow + c);
-                v.x = __fmaf_rn(alpha, acc[i][4 * h + 0], v.x);
-                v.y = __fmaf_rn(alpha, acc[i][4 * h + 1], v.y);
-                v.z = __fmaf_rn(alpha, acc[i][4 * h + 2], v.z);
-                v.w = __fmaf_rn(alpha, acc[i][4 * h + 3], v.w);
+                v.x = __fmaf_rn(alpha, o[0], v.x);
+                v.y = __fmaf_rn(alpha, o[1], v.y);
+                v.z = __fmaf_rn(alpha, o[2], v.z);
+                v.w = __fmaf_rn(alpha, o[3], v.w);
                 *reinterpret_cast<float4*>(crow + c) = v;
             } else {
 #pragma unroll
                 for (int j = 0; j < 4; j++)
-                    if (c + j < N) crow[c + j] = __fmaf_rn(alpha, acc[i][4 * h + j], crow[c + j]);
+                    if (c + j < N) crow[c + j] = __fmaf_rn(alpha, o[j], crow[c + j]);
             }
         }
     }
