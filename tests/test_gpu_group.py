@@ -220,3 +220,70 @@ def test_group_rejects_overlapping_buffers(B):
     B.scalesweep_quantize_group(ok, B.NVFP4_IN_BF16, 0, 256.0, S, None, wsb)
     torch.cuda.synchronize()
     assert S[0].item() == 0.0 and not torch.any(codes & 0x77).item()
+
+
+def test_group_output_guard_bytes_untouched(B):
+    """Outputs of a ragged group carved from one buffer with 4 KiB guards between
+    them: every guard byte survives (the 256-segment padding of each tensor's
+    range is never written)."""
+    shapes = [(37, 48), (130, 192), (1, 64)]
+    xs, ws, strides = make_group(torch.bfloat16, 1, seed=7, shapes=shapes, row_weights=())
+    G = 4096
+    sizes = []
+    for r, c in shapes:
+        sizes += [r * c // 2, r * c // 16, B.swizzled_bytes(r, c)]
+    offs, pos = [], G
+    for n in sizes:
+        pos = (pos + 15) // 16 * 16
+        offs.append(pos)
+        pos += n + G
+    buf = torch.full((pos,), 0xAB, dtype=torch.uint8, device=DEV)
+    views = [buf[o:o + n] for o, n in zip(offs, sizes)]
+    codes = [views[3 * i].view(r, c // 2) for i, (r, c) in enumerate(shapes)]
+    sfl = [views[3 * i + 1].view(r, c // 16) for i, (r, c) in enumerate(shapes)]
+    sfs = [views[3 * i + 2] for i in range(len(shapes))]
+    dx = [x.to(DEV) for x in xs]
+    dw = [w.to(DEV) for w in ws]
+    desc = B.group_descriptors(dx, dw, strides, codes, sfl, sfs)
+    S = torch.empty(len(shapes), device=DEV)
+    wsb = torch.empty(B.scalesweep_quantize_group_workspace(), dtype=torch.uint8, device=DEV)
+    B.scalesweep_quantize_group(desc, B.NVFP4_IN_BF16, 1, 256.0, S, None, wsb)
+    torch.cuda.synchronize()
+    mask = torch.ones(pos, dtype=torch.bool, device=DEV)
+    for o, n in zip(offs, sizes):
+        mask[o:o + n] = False
+    assert torch.all(buf[mask] == 0xAB)
+    for i, x in enumerate(dx):
+        _, _, o1 = per_tensor(B, x, dw[i], strides[i], 1)
+        assert torch.equal(codes[i], o1["codes"]) and torch.equal(sfl[i], o1["sf_linear"])
+        assert torch.equal(sfs[i], o1["sf_swizzled"])
+
+
+def test_group_dynamic_in_cuda_graph(B):
+    """The grouped call (workspace memset + cooperative launch) captured in a
+    CUDA graph and replayed gives the eager results; the library neither
+    allocates nor synchronises, so it can be captured."""
+    xs, ws, strides = make_group(torch.bfloat16, 1, seed=8, shapes=[(300, 512), (64, 80), (1024, 256)])
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, 1)
+    outs2 = [B.empty_outputs(x.shape[0], x.shape[1], 16, device=DEV, linear=True, swizzled=True) for x in xs]
+    desc = B.group_descriptors(dev_x, dev_w, strides, [o["codes"] for o in outs2], [o["sf_linear"] for o in outs2],
+                               [o["sf_swizzled"] for o in outs2])
+    S2 = torch.zeros(len(xs), device=DEV)
+    st2 = torch.zeros(1, dtype=torch.int32, device=DEV)
+    wsb = torch.empty(B.scalesweep_quantize_group_workspace(), dtype=torch.uint8, device=DEV)
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        B.scalesweep_quantize_group(desc, B.NVFP4_IN_BF16, 1, 256.0, S2, st2, wsb, stream=s)   # warm-up
+    torch.cuda.synchronize()
+    with torch.cuda.graph(g, stream=s):
+        B.scalesweep_quantize_group(desc, B.NVFP4_IN_BF16, 1, 256.0, S2, st2, wsb, stream=s)
+    for _ in range(2):
+        for o in outs2:
+            o["codes"].zero_()
+        g.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(S2, S) and st2.item() == 0
+        for a, b in zip(outs, outs2):
+            for k in ("codes", "sf_linear", "sf_swizzled"):
+                assert torch.equal(a[k], b[k])
