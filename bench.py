@@ -540,6 +540,12 @@ def run_kernel_case(args):
                                                     o["sf_swizzled"]),
         "sweep_mse": lambda: B.scalesweep_quantize(x, args.block, S, 0, None, 0, *win, o["codes"], o["sf_linear"],
                                                    o["sf_swizzled"]),
+        "sweep_wmse_tight": lambda: B.scalesweep_quantize(x, args.block, S, 1, w, 0, B.NVFP4_WINDOW_TIGHT,
+                                                          B.NVFP4_WINDOW_TIGHT, o["codes"], o["sf_linear"],
+                                                          o["sf_swizzled"]),
+        "sweep_mse_tight": lambda: B.scalesweep_quantize(x, args.block, S, 0, None, 0, B.NVFP4_WINDOW_TIGHT,
+                                                         B.NVFP4_WINDOW_TIGHT, o["codes"], o["sf_linear"],
+                                                         o["sf_swizzled"]),
         "absmax": lambda: B.absmax_quantize(x, args.block, S, o["codes"], o["sf_linear"], o["sf_swizzled"]),
         "four_six": lambda: B.four_over_six_quantize(x, args.block, S, 1, w, 0, o["codes"], o["sf_linear"],
                                                      o["sf_swizzled"]),
@@ -843,6 +849,7 @@ def main():
     ap.add_argument("--kernel-case", default=None,
                     choices=["sweep_wmse", "sweep_mse", "absmax", "four_six", "dequant", "amax", "mse_two_launch",
                              "sweep_wmse_group", "wmse_group_dynamic", "group_layer", "group_layer_static",
+                             "sweep_wmse_tight", "sweep_mse_tight",
                              "layer_per_tensor_static", "group_layer_linear", "group_layer_static_linear",
                              "mse_fused", "wmse_fused"])
     ap.add_argument("--rows", type=int, default=16384)

@@ -63,6 +63,16 @@ typedef enum { NVFP4_SF_LINEAR = 1, NVFP4_SF_SWIZZLED = 2 } nvfp4_sf_layout;
 
 /* Pass as win_lo and win_hi to use the paper's window (Sec. 4.2.2). */
 #define NVFP4_WINDOW_DEFAULT INT_MIN
+/* Pass as win_lo and win_hi for the paper's window tightened per block without
+ * changing the result (the exact-window refinement of Sec. 4.2.2): the upper end
+ * drops every code c >= 16 with 3.5 v_c > max|y| (Lemma 4.1: such an s never
+ * beats s/2, which is code c - 8 and stays in the window; 3.5 v_c is exact in
+ * fp32; below code 16 half a scale need not be a code), and for MSE with block
+ * 16 the lower end is the
+ * per-mantissa bound of Table 3 (I0 - 2, or I0 - 3 for mantissas 000 and 111;
+ * applied for I0 in 16..120, where the ceiling stays normal and Lemma 4.3's
+ * 11/7 s <= 448 holds).  A warp runs as many candidates as its widest block. */
+#define NVFP4_WINDOW_TIGHT (INT_MIN + 1)
 
 /* Human-readable name of a status code (static storage). */
 const char* nvfp4_status_string(nvfp4_status st);
@@ -124,6 +134,7 @@ nvfp4_status nvfp4_global_scale_noalloc(const void* x, nvfp4_dtype dt, int64_t n
  *                 NVFP4_WINDOW_DEFAULT: [-3, 7] for MSE with block 16 (Lemma 4.3),
  *                 [-8, 7] otherwise (WMSE: empirical s_base/2; blocks of 32/64:
  *                 the paper gives no window).  (-126, 126) is the exhaustive sweep.
+ *                 Both NVFP4_WINDOW_TIGHT: the default window tightened per block.
  *   codes         [rows, cols/2] packed nibbles, 8-byte aligned.
  *   sf_linear     optional [rows, cols/block] scale codes.
  *   sf_swizzled   optional 128x4-atom scale layout (block 16 only).

@@ -19,6 +19,7 @@ NVFP4_IN_BF16, NVFP4_IN_F32 = 0, 1
 NVFP4_OBJ_MSE, NVFP4_OBJ_WMSE = 0, 1
 NVFP4_SF_LINEAR, NVFP4_SF_SWIZZLED = 1, 2
 NVFP4_WINDOW_DEFAULT = -(2 ** 31)
+NVFP4_WINDOW_TIGHT = -(2 ** 31) + 1
 
 STATUS = {0: "NVFP4_OK", 1: "NVFP4_ERR_INVALID_ARG", 2: "NVFP4_ERR_UNSUPPORTED", 3: "NVFP4_ERR_ALIGNMENT",
           4: "NVFP4_ERR_RANGE", 5: "NVFP4_ERR_CUDA"}

@@ -103,7 +103,12 @@ nvfp4_status quantize_common(int method, const void* x, nvfp4_dtype dt, int64_t 
     nvfp4_status st = check_shape(rows, cols, block, &sh);
     if (st != NVFP4_OK) return st;
     if (sf_swizzled && block != 16) return NVFP4_ERR_UNSUPPORTED;
+    int tight = 0;
     if (method == 0) {
+        if (win_lo == NVFP4_WINDOW_TIGHT && win_hi == NVFP4_WINDOW_TIGHT) {
+            tight = 1 | ((obj == NVFP4_OBJ_MSE && block == 16) ? 2 : 0);
+            win_lo = win_hi = NVFP4_WINDOW_DEFAULT;
+        }
         if (win_lo == NVFP4_WINDOW_DEFAULT && win_hi == NVFP4_WINDOW_DEFAULT) {
             win_lo = (obj == NVFP4_OBJ_MSE && block == 16) ? -3 : -8;   // Lemma 4.3 / Sec. 4.2.2
             win_hi = 7;                                                 // Lemma 4.2, alpha = 12/7
@@ -172,6 +177,7 @@ nvfp4_status quantize_common(int method, const void* x, nvfp4_dtype dt, int64_t 
     p.narrow = sh.narrow;
     p.win_lo = win_lo;
     p.win_hi = win_hi;
+    p.tight = tight;
     p.codes = codes;
     p.sf_linear = sf_linear;
     p.sf_swizzled = sf_swizzled;

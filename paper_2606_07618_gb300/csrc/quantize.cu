@@ -65,7 +65,7 @@ FastDiv make_fast_div(uint32_t d) {
 
 void prepare_quant_params(QuantParams& p, int method, int obj, int block, bool* fix) {
     const int def_lo = (obj == 0 && block == 16) ? -3 : -8;
-    *fix = (method != 0) || (p.win_lo == def_lo && p.win_hi == 7);
+    *fix = (method != 0) || (p.win_lo == def_lo && p.win_hi == 7 && !p.tight);
     p.need_rowcol = (p.sf_swizzled != nullptr) || (obj == 1);
     if (p.narrow) p.kb_div = make_fast_div((uint32_t)p.kb);
 }

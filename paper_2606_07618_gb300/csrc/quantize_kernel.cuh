@@ -365,8 +365,18 @@ __global__ void __launch_bounds__(256, NVFP4_QMINB) quantize_kernel(QuantParams 
                 }
                 bestc = I0 + FIX_LO + bk;
             } else {
-                const int clo = min(max(I0 + p.win_lo, 1), 126);
-                const int chi = min(max(I0 + p.win_hi, 1), 126);
+                int lo_off = p.win_lo;
+                if ((p.tight & 2) && I0 >= 16 && I0 <= 120) {
+                    const int b = I0 & 7;                       // Table 3: ceil(4/5 s) is 2 or 3 codes down
+                    lo_off = (b == 0 || b == 7) ? -3 : -2;
+                }
+                const int clo = min(max(I0 + lo_off, 1), 126);
+                int chi = min(max(I0 + p.win_hi, 1), 126);
+                if (p.tight & 1) {     // Lemma 4.1: 3.5 v_c > m never beats v_c / 2 = code c - 8 (c >= 16)
+                    while (chi > clo && chi >= 16 &&
+                           __fmul_rn(3.5f, f16bits_to_f32((uint16_t)(tab[chi + kTabOff].nv ^ 0x8000u))) > m)
+                        chi--;
+                }
                 const int n = zero ? 0 : chi - clo + 1;
                 const int nmax = __reduce_max_sync(0xffffffffu, (unsigned)n);
                 bestc = clo;
