@@ -232,6 +232,21 @@ nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int co
                                        void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * Self-test of the bounded device waits (failure detection; the paper has no
+ * counterpart).  Runs scalesweep_quantize_dynamic (which = 0: bf16 x, block
+ * 16, MSE, default window) or scalesweep_quantize_group with a dynamic scale
+ * (which = 1: x as its one tensor, MSE) with the wait's arrival target raised
+ * past what the launch can reach, so every device wait gives up after its
+ * limit (about a second): bit 1 is OR-ed into *status_dev (required here), the
+ * waiting warps return without writing codes or scales, and the CUDA context
+ * stays usable.  Arguments and buffers as in those calls; workspace of
+ * max(nvfp4_dynamic_workspace(), scalesweep_quantize_group_workspace()) bytes.
+ */
+nvfp4_status nvfp4_selftest_wait_timeout(int which, const void* x, int64_t rows, int64_t cols, float* S,
+                                         int* status_dev, void* workspace, size_t ws_bytes, uint8_t* codes,
+                                         uint8_t* sf_linear, void* stream);
+
+/*
  * AbsMax quantisation with the global scale computed in the same launch, as
  * scalesweep_quantize_dynamic (baseline for the fused dynamic path).
  */

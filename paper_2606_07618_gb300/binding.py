@@ -70,6 +70,7 @@ def lib() -> ctypes.CDLL:
         L.absmax_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, p, p, p, sz, p, p, p, p, p]
         L.scalesweep_quantize_group_workspace.argtypes, L.scalesweep_quantize_group_workspace.restype = [], sz
         L.scalesweep_quantize_group.argtypes = [ctypes.POINTER(GroupTensor), i, i, i, f, p, p, p, sz, p]
+        L.nvfp4_selftest_wait_timeout.argtypes = [i, p, i64, i64, p, p, p, sz, p, p, p]
         L.nvfp4_optimal_scale.argtypes = [p, i, i64, i64, i, p, i, p, i64, p, p, p, p, p]
         L.nvfp4_ldlq_prepare_workspace.argtypes, L.nvfp4_ldlq_prepare_workspace.restype = [i64], sz
         L.nvfp4_ldlq_prepare.argtypes = [p, i64, f, p, p, p, p, p, sz, p]
@@ -78,7 +79,7 @@ def lib() -> ctypes.CDLL:
         for fn in ("nvfp4_global_scale", "nvfp4_global_scale_noalloc", "scalesweep_quantize", "absmax_quantize",
                    "four_over_six_quantize", "nvfp4_dequantize", "scalesweep_quantize_dynamic",
                    "absmax_quantize_dynamic", "nvfp4_optimal_scale", "nvfp4_ldlq_prepare", "ldlq_quantize",
-                   "scalesweep_quantize_group"):
+                   "scalesweep_quantize_group", "nvfp4_selftest_wait_timeout"):
             getattr(L, fn).restype = i
         _lib = L
     return _lib
@@ -214,6 +215,16 @@ def scalesweep_quantize_group(desc, dtype: int, objective: int, fp8_div: float, 
     rc = lib().scalesweep_quantize_group(desc, len(desc), int(dtype), int(objective), float(fp8_div), _ptr(S),
                                          _ptr(status), _ptr(workspace), ws_bytes, _stream(stream))
     _check("scalesweep_quantize_group", rc)
+
+
+def nvfp4_selftest_wait_timeout(which: int, x, S, status, workspace, codes, sf_linear, stream=None):
+    """Makes the device waits of the dynamic-scale sweep (which = 0) or of the
+    grouped launch (which = 1) run out; status bit 1 reports it."""
+    rows, cols = x.shape
+    ws_bytes = workspace.numel() * workspace.element_size()
+    rc = lib().nvfp4_selftest_wait_timeout(int(which), _ptr(x), rows, cols, _ptr(S), _ptr(status), _ptr(workspace),
+                                           ws_bytes, _ptr(codes), _ptr(sf_linear), _stream(stream))
+    _check("nvfp4_selftest_wait_timeout", rc)
 
 
 def nvfp4_optimal_scale(x, block: int, S, objective: int, w, w_row_stride: int, s_opt, loss_opt, fp8_code=None,

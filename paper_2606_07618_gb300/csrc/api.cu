@@ -91,6 +91,7 @@ struct DynArgs {
     int* status_dev;
     void* workspace;
     size_t ws_bytes;
+    unsigned wait_extra;     // 0 except in nvfp4_selftest_wait_timeout
 };
 
 nvfp4_status quantize_common(int method, const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
@@ -188,6 +189,7 @@ nvfp4_status quantize_common(int method, const void* x, nvfp4_dtype dt, int64_t 
     p.part_max = nullptr;
     p.part_bad = nullptr;
     p.barrier = nullptr;
+    p.wait_extra = 0;
     const int dti = dt == NVFP4_IN_BF16 ? 0 : 1, obji = obj == NVFP4_OBJ_WMSE ? 1 : 0;
     cudaError_t e;
     if (dyn) {
@@ -197,6 +199,7 @@ nvfp4_status quantize_common(int method, const void* x, nvfp4_dtype dt, int64_t 
         p.part_max = static_cast<float*>(dyn->workspace);
         p.part_bad = reinterpret_cast<int*>(p.part_max + kAmaxParts);
         p.barrier = reinterpret_cast<unsigned*>(p.part_bad + kAmaxParts);
+        p.wait_extra = dyn->wait_extra;
         e = launch_quantize_dynamic(p, dti, method, obji, block, sms, static_cast<cudaStream_t>(stream));
     } else {
         e = launch_quantize(p, dti, method, obji, block, sms, static_cast<cudaStream_t>(stream));
@@ -265,7 +268,7 @@ nvfp4_status scalesweep_quantize_dynamic(const void* x, nvfp4_dtype dt, int64_t 
                                          int win_lo, int win_hi, float* S_out, int* status_dev, void* workspace,
                                          size_t ws_bytes, uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled,
                                          float* block_loss, void* stream) {
-    const DynArgs d{fp8_div, S_out, status_dev, workspace, ws_bytes};
+    const DynArgs d{fp8_div, S_out, status_dev, workspace, ws_bytes, 0};
     return quantize_common(0, x, dt, rows, cols, block, nullptr, obj, w, w_row_stride, win_lo, win_hi, codes,
                            sf_linear, sf_swizzled, block_loss, stream, &d);
 }
@@ -274,9 +277,10 @@ static_assert(kGroupMax == NVFP4_GROUP_MAX, "group descriptor count");
 
 size_t scalesweep_quantize_group_workspace(void) { return kGroupWorkspace; }
 
-nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt,
-                                       nvfp4_objective obj, float fp8_div, float* S, int* status_dev,
-                                       void* workspace, size_t ws_bytes, void* stream) {
+namespace {
+nvfp4_status group_common(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt, nvfp4_objective obj,
+                          float fp8_div, float* S, int* status_dev, void* workspace, size_t ws_bytes, void* stream,
+                          unsigned wait_extra) {
     if (dt != NVFP4_IN_BF16 && dt != NVFP4_IN_F32) return NVFP4_ERR_INVALID_ARG;
     if (obj != NVFP4_OBJ_MSE && obj != NVFP4_OBJ_WMSE) return NVFP4_ERR_INVALID_ARG;
     if (!tensors || count < 1 || count > NVFP4_GROUP_MAX || !S) return NVFP4_ERR_INVALID_ARG;
@@ -387,16 +391,38 @@ nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int co
     p.status_dev = status_dev;
     p.amax_bits = dyn ? static_cast<unsigned*>(workspace) : nullptr;
     p.arrived = dyn ? static_cast<unsigned*>(workspace) + kGroupMax : nullptr;
+    p.wait_extra = wait_extra;
     const cudaError_t e = launch_quantize_group(p, rows, dt == NVFP4_IN_BF16 ? 0 : 1, obj == NVFP4_OBJ_WMSE ? 1 : 0,
                                                 sms, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
+}
+}  // namespace
+
+nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt,
+                                       nvfp4_objective obj, float fp8_div, float* S, int* status_dev,
+                                       void* workspace, size_t ws_bytes, void* stream) {
+    return group_common(tensors, count, dt, obj, fp8_div, S, status_dev, workspace, ws_bytes, stream, 0);
+}
+
+nvfp4_status nvfp4_selftest_wait_timeout(int which, const void* x, int64_t rows, int64_t cols, float* S,
+                                         int* status_dev, void* workspace, size_t ws_bytes, uint8_t* codes,
+                                         uint8_t* sf_linear, void* stream) {
+    if ((which != 0 && which != 1) || !status_dev || rows <= 0 || cols <= 0) return NVFP4_ERR_INVALID_ARG;
+    if (which == 0) {
+        const DynArgs d{256.0f, S, status_dev, workspace, ws_bytes, 1};
+        return quantize_common(0, x, NVFP4_IN_BF16, rows, cols, 16, nullptr, NVFP4_OBJ_MSE, nullptr, 0,
+                               NVFP4_WINDOW_DEFAULT, NVFP4_WINDOW_DEFAULT, codes, sf_linear, nullptr, nullptr, stream,
+                               &d);
+    }
+    const nvfp4_group_tensor t{x, rows, cols, nullptr, 0, codes, sf_linear, nullptr};
+    return group_common(&t, 1, NVFP4_IN_BF16, NVFP4_OBJ_MSE, 256.0f, S, status_dev, workspace, ws_bytes, stream, 1);
 }
 
 nvfp4_status absmax_quantize_dynamic(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,
                                      float fp8_div, float* S_out, int* status_dev, void* workspace, size_t ws_bytes,
                                      uint8_t* codes, uint8_t* sf_linear, uint8_t* sf_swizzled, float* block_loss,
                                      void* stream) {
-    const DynArgs d{fp8_div, S_out, status_dev, workspace, ws_bytes};
+    const DynArgs d{fp8_div, S_out, status_dev, workspace, ws_bytes, 0};
     return quantize_common(1, x, dt, rows, cols, block, nullptr, NVFP4_OBJ_MSE, nullptr, 0, 0, 0, codes, sf_linear,
                            sf_swizzled, block_loss, stream, &d);
 }

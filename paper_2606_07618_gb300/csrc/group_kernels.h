@@ -38,6 +38,7 @@ struct GroupParams {
     int* status_dev;
     unsigned* amax_bits;       // [count] workspace, zeroed before the launch
     unsigned* arrived;         // [count] workspace, zeroed before the launch
+    unsigned wait_extra;       // added to the arrival target; 0 except in the wait self-test
 };
 
 constexpr size_t kGroupWorkspace = 256;   // amax_bits + arrived for kGroupMax tensors

@@ -34,6 +34,7 @@ struct QuantParams {
     float* part_max;
     int* part_bad;
     unsigned* barrier;
+    unsigned wait_extra;     // added to the barrier's arrival target; 0 except in the wait self-test
 };
 
 // dtype 0 bf16 / 1 f32; method 0 ScaleSweep / 1 AbsMax / 2 four-over-six;

@@ -27,8 +27,9 @@
 // counts itself in arrived[a] (acquire-release); the last to arrive writes
 // S[a].  A sweep warp entering tensor t waits until all NA reduction warps
 // have arrived for t.  Reduction warps never wait, and the grid is resident
-// (cooperative launch), so every wait ends; each is bounded anyway (status bit
-// 1, the warp stops).  Tensors are processed in ascending size, so the first
+// (cooperative launch), so every wait ends; each is bounded anyway by the
+// global timer (1 s; status bit 1, the warp stops).  p.wait_extra raises the
+// arrival target: 0 in every real call, the wait self-test uses it.  Tensors are processed in ascending size, so the first
 // reduction, the only one no sweep hides, is the smallest.
 #include <atomic>
 
@@ -302,7 +303,7 @@ __global__ void __launch_bounds__(DYN ? kSweepThreads + 32 : kSweepThreads, NVFP
             int timeout = 0;
             if (lane == 0) {
                 const unsigned long long t0 = global_ns();
-                while (ld_acquire_u32(p.arrived + t) < gridDim.x) {
+                while (ld_acquire_u32(p.arrived + t) < gridDim.x + p.wait_extra) {
                     if (global_ns() - t0 > kGroupWaitNs) {
                         timeout = 1;
                         break;

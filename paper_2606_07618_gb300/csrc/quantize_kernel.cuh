@@ -159,9 +159,17 @@ constexpr int kCandUnroll = NVFP4_CAND_UNROLL;
 // max |x| of its grid-stride share into one partial, all CTAs meet at a grid
 // barrier (cooperative launch, so all are resident; the counter is zeroed by
 // the host before the launch), then each CTA folds all partials into the same
-// S = fl(amax / fl(6 D)).  The barrier wait is bounded: on timeout the kernel
-// sets bit 1 of the status word and returns without writing outputs.
-constexpr unsigned kBarrierSpinLimit = 1u << 24;
+// S = fl(amax / fl(6 D)).  The barrier wait is bounded by the global timer
+// (1 s): on timeout the kernel sets bit 1 of the status word and returns
+// without writing outputs.  p.wait_extra raises the arrival target (0 in every
+// real call; the wait self-test uses it to make the wait run out).
+constexpr unsigned long long kBarrierWaitNs = 1000000000ull;
+
+__device__ __forceinline__ unsigned long long globaltimer_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
 
 __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
     unsigned v;
@@ -223,14 +231,14 @@ __device__ __forceinline__ bool dynamic_scale(const QuantParams& p, float& S_out
         p.part_bad[blockIdx.x] = b;
         __threadfence();
         atomicAdd(p.barrier, 1u);
-        unsigned spins = 0;
+        const unsigned long long t0 = globaltimer_ns();
         int timeout = 0;
-        while (ld_acquire_u32(p.barrier) < gridDim.x) {
-            if (++spins > kBarrierSpinLimit) {
+        while (ld_acquire_u32(p.barrier) < gridDim.x + p.wait_extra) {
+            if (globaltimer_ns() - t0 > kBarrierWaitNs) {
                 timeout = 1;
                 break;
             }
-            __nanosleep(64);
+            __nanosleep(128);
         }
         s_timeout = timeout;
     }

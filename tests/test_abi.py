@@ -30,7 +30,8 @@ def test_header_declares_the_api():
         "scalesweep_quantize", "absmax_quantize", "four_over_six_quantize", "nvfp4_dequantize",
         "nvfp4_dynamic_workspace", "scalesweep_quantize_dynamic", "absmax_quantize_dynamic",
         "nvfp4_optimal_scale", "nvfp4_ldlq_prepare_workspace", "nvfp4_ldlq_prepare", "nvfp4_ldlq_workspace",
-        "ldlq_quantize", "scalesweep_quantize_group_workspace", "scalesweep_quantize_group"])
+        "ldlq_quantize", "scalesweep_quantize_group_workspace", "scalesweep_quantize_group",
+        "nvfp4_selftest_wait_timeout"])
 
 
 def test_library_exports_every_declared_symbol(L):
@@ -156,3 +157,8 @@ def test_group_validation_without_gpu(L):
     assert g(desc(every={"w": FAKE + 0x4000004}), obj=1) == 3
     assert g(desc(every={"w": FAKE + 0x4000000, "w_row_stride": 8}), obj=1) == 1
     assert g(desc({"rows": 2 ** 40, "cols": 2 ** 40})) == 4
+    st_test = lambda which=0, status=st, rows=4: L.nvfp4_selftest_wait_timeout(
+        which, FAKE, rows, 64, S, status, ws, 1 << 12, FAKE + 0x1000000, FAKE + 0x2000000, None)
+    assert st_test(which=2) == 1
+    assert st_test(status=None) == 1                 # the status word is how the timeout is seen
+    assert st_test(rows=0) == 1
