@@ -125,6 +125,7 @@ __global__ void __launch_bounds__(256) potrf_kernel(float* A, int64_t n, int64_t
     __shared__ float piv[kP];
     const int r0 = (threadIdx.x >> 4) * 4, c0 = (threadIdx.x & 15) * 4;
     float t[4][4];
+    float x[4][4];                                   // X = M^-1 (unit lower), built alongside
 #pragma unroll
     for (int di = 0; di < 4; di++)
 #pragma unroll
@@ -133,7 +134,12 @@ __global__ void __launch_bounds__(256) potrf_kernel(float* A, int64_t n, int64_t
             float v = (i < nb && l < nb && l <= i) ? A[(k0 + i) * n + k0 + l] : 0.0f;
             if (i >= nb && i == l) v = 1.0f;
             t[di][dl] = v;
+            x[di][dl] = i == l ? 1.0f : 0.0f;
         }
+    // Step j: column j of the reduced matrix gives the pivot and the multipliers
+    // m_ij = a_ij / p_j (= M's column j); the trailing update and the inverse's
+    // row operation X_i -= m_ij X_j (row j of X is final at step j) share one
+    // barrier.  Per entry the inverse sees its updates in the order k = 0, 1, ...
     int bad = 0;
     for (int j = 0; j < kP; j++) {
         const int b = j & 1;
@@ -143,6 +149,14 @@ __global__ void __launch_bounds__(256) potrf_kernel(float* A, int64_t n, int64_t
                 const int q = j - c0;
                 const float v = q == 0 ? t[di][0] : q == 1 ? t[di][1] : q == 2 ? t[di][2] : t[di][3];
                 colv[b][r0 + di] = v;
+            }
+        }
+        if (r0 <= j && j < r0 + 4) {                 // row j of X
+#pragma unroll
+            for (int dc = 0; dc < 4; dc++) {
+                const int q = j - r0;
+                const float v = q == 0 ? x[0][dc] : q == 1 ? x[1][dc] : q == 2 ? x[2][dc] : x[3][dc];
+                rowv[b][c0 + dc] = v;
             }
         }
         __syncthreads();
@@ -155,7 +169,9 @@ __global__ void __launch_bounds__(256) potrf_kernel(float* A, int64_t n, int64_t
         const float ip = __frcp_rn(p);
         const float4 ci = *reinterpret_cast<const float4*>(&colv[b][r0]);
         const float4 cl = *reinterpret_cast<const float4*>(&colv[b][c0]);
+        const float4 xj = *reinterpret_cast<const float4*>(&rowv[b][c0]);
         const float civ[4] = {ci.x, ci.y, ci.z, ci.w}, clv[4] = {cl.x, cl.y, cl.z, cl.w};
+        const float xjv[4] = {xj.x, xj.y, xj.z, xj.w};
 #pragma unroll
         for (int di = 0; di < 4; di++) {
             const int i = r0 + di;
@@ -164,6 +180,7 @@ __global__ void __launch_bounds__(256) potrf_kernel(float* A, int64_t n, int64_t
             for (int dl = 0; dl < 4; dl++) {
                 const int l = c0 + dl;
                 if (i > j && l > j && l <= i) t[di][dl] = __fmaf_rn(-aij, clv[dl], t[di][dl]);
+                if (i > j && l <= j) x[di][dl] = __fmaf_rn(-aij, xjv[dl], x[di][dl]);
             }
         }
     }
@@ -174,40 +191,6 @@ __global__ void __launch_bounds__(256) potrf_kernel(float* A, int64_t n, int64_t
 #pragma unroll
         for (int dl = 0; dl < 4; dl++)
             if (c0 + dl < r0 + di) t[di][dl] = __fmul_rn(t[di][dl], __frcp_rn(piv[c0 + dl]));
-    // X = M^-1 (unit lower), tile x: row k of X is final at step k
-    float x[4][4];
-#pragma unroll
-    for (int di = 0; di < 4; di++)
-#pragma unroll
-        for (int dc = 0; dc < 4; dc++) x[di][dc] = (r0 + di == c0 + dc) ? 1.0f : 0.0f;
-    for (int k = 0; k < kP; k++) {
-        const int b = k & 1;
-        if (c0 <= k && k < c0 + 4) {                 // column k of M
-#pragma unroll
-            for (int di = 0; di < 4; di++) {
-                const int q = k - c0;
-                const float v = q == 0 ? t[di][0] : q == 1 ? t[di][1] : q == 2 ? t[di][2] : t[di][3];
-                colv[b][r0 + di] = v;
-            }
-        }
-        if (r0 <= k && k < r0 + 4) {                 // row k of X
-#pragma unroll
-            for (int dc = 0; dc < 4; dc++) {
-                const int q = k - r0;
-                const float v = q == 0 ? x[0][dc] : q == 1 ? x[1][dc] : q == 2 ? x[2][dc] : x[3][dc];
-                rowv[b][c0 + dc] = v;
-            }
-        }
-        __syncthreads();
-        const float4 mi = *reinterpret_cast<const float4*>(&colv[b][r0]);
-        const float4 xk = *reinterpret_cast<const float4*>(&rowv[b][c0]);
-        const float miv[4] = {mi.x, mi.y, mi.z, mi.w}, xkv[4] = {xk.x, xk.y, xk.z, xk.w};
-#pragma unroll
-        for (int di = 0; di < 4; di++)
-#pragma unroll
-            for (int dc = 0; dc < 4; dc++)
-                if (r0 + di > k && c0 + dc <= k) x[di][dc] = __fmaf_rn(-miv[di], xkv[dc], x[di][dc]);
-    }
 #pragma unroll
     for (int di = 0; di < 4; di++)
 #pragma unroll
