@@ -86,19 +86,18 @@ def lib() -> ctypes.CDLL:
 
 
 def _ptr(t):
-    if t is None:
-        return None
-    if isinstance(t, int):
-        return ctypes.c_void_p(t)
-    return ctypes.c_void_p(t.data_ptr())
+    # plain ints: ctypes converts them for c_void_p parameters without an object
+    if t is None or isinstance(t, int):
+        return t
+    return t.data_ptr()
 
 
 def _stream(stream):
     if stream is None:
-        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+        return torch.cuda.current_stream().cuda_stream
     if isinstance(stream, torch.cuda.Stream):
-        return ctypes.c_void_p(stream.cuda_stream)
-    return ctypes.c_void_p(int(stream))
+        return stream.cuda_stream
+    return int(stream)
 
 
 def _dtype(x) -> int:
