@@ -327,6 +327,12 @@ nvfp4_status nvfp4_dequantize(const uint8_t* codes, const uint8_t* sf, nvfp4_sf_
  *           factorization then).
  *   workspace   device bytes, at least nvfp4_ldlq_prepare_workspace(n).
  * Cost: n^3/3 fp32 multiply-adds (blocked Cholesky, 64-wide panels).
+ * The factorization's critical chain runs on a high-priority stream the library
+ * creates on the first call on a device and keeps (with four events) for the
+ * process; it is forked from and joined back into `stream`, so the call stays
+ * ordered on `stream` and can be captured in a CUDA graph -- make the first
+ * call on each device outside a capture.  Concurrent calls on one device are
+ * serialised while they enqueue.
  */
 size_t nvfp4_ldlq_prepare_workspace(int64_t n);
 nvfp4_status nvfp4_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* perm, float* U, float* D,

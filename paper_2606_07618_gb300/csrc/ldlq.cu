@@ -21,6 +21,7 @@
 // What = fl(fl(q*v_c)*S); a zero-scale block or an unusable S gives signed
 // zeros; an exactly zero y takes the +0 code.
 #include <atomic>
+#include <mutex>
 
 #include <cuda_bf16.h>
 
@@ -571,6 +572,39 @@ size_t ldlq_prepare_workspace(int64_t n) {
     return (size_t)((n * 4 + 255) / 256 * 256) + 256 + (size_t)kP * kP * 4;
 }
 
+// Stream and events of the factorization's look-ahead, one set per device,
+// created on the first prepare call on that device and kept for the process.
+// The critical chain (diagonal factor, panel solve, next block column) runs on
+// `crit`, created with the device's highest priority so its CTAs are placed
+// before the pending tiles of the bulk update on the caller's stream.  The
+// mutex serialises enqueueing, so the record/wait pairs of two concurrent calls
+// cannot interleave.
+struct LookAhead {
+    cudaStream_t crit = nullptr;
+    cudaEvent_t fork = nullptr, panel_done = nullptr, rest_done = nullptr, crit_done = nullptr;
+};
+
+cudaError_t lookahead_for_current_device(LookAhead** out, std::unique_lock<std::mutex>* lock) {
+    static std::mutex mu;
+    static LookAhead state[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    *lock = std::unique_lock<std::mutex>(mu);
+    LookAhead& la = state[dev];
+    if (!la.crit) {
+        int least = 0, greatest = 0;
+        if ((e = cudaDeviceGetStreamPriorityRange(&least, &greatest)) != cudaSuccess) return e;
+        if ((e = cudaStreamCreateWithPriority(&la.crit, cudaStreamNonBlocking, greatest)) != cudaSuccess) return e;
+        cudaEvent_t* evs[4] = {&la.fork, &la.panel_done, &la.rest_done, &la.crit_done};
+        for (cudaEvent_t* ev : evs)
+            if ((e = cudaEventCreateWithFlags(ev, cudaEventDisableTiming)) != cudaSuccess) return e;
+    }
+    *out = &la;
+    return cudaSuccess;
+}
+
 cudaError_t launch_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* perm, float* U, float* D,
                                 int* status, void* ws, int sms, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
@@ -584,20 +618,46 @@ cudaError_t launch_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* 
     gather_h_kernel<<<rg, 256, 0, s>>>(H, n, perm, lam, U);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
+    // Look-ahead: the trailing update of panel k is split into the next panel's
+    // block column (on the high-priority stream, with the next diagonal factor
+    // and panel solve) and the rest (on `s`, overlapping them).  The two
+    // updates of one block column from different panels are ordered by events.
+    LookAhead* la = nullptr;
+    std::unique_lock<std::mutex> lock;
+    e = lookahead_for_current_device(&la, &lock);
+    if (e != cudaSuccess) return e;
+    cudaStream_t c = la->crit;
+    if ((e = cudaEventRecord(la->fork, s)) != cudaSuccess) return e;
+    if ((e = cudaStreamWaitEvent(c, la->fork, 0)) != cudaSuccess) return e;
     for (int64_t k0 = 0; k0 < n; k0 += kP) {
         const int nb = (int)imin64(kP, n - k0);
-        potrf_kernel<<<1, 256, 0, s>>>(U, n, k0, nb, Linv, status);
+        potrf_kernel<<<1, 256, 0, c>>>(U, n, k0, nb, Linv, status);
         const int64_t rest = n - k0 - nb;
         if (rest > 0) {
             const unsigned tg = (unsigned)imin64((rest + 7) / 8, (int64_t)sms * 8);
-            trsm_kernel<<<tg, 256, 0, s>>>(U, n, k0, nb, Linv);
-            float* P = U + (k0 + nb) * n + k0;
-            e = launch_gemm<false, true, true>(U + (k0 + nb) * n + k0 + nb, n, P, n, P, n, rest, rest, nb, -1.0f, s);
+            trsm_kernel<<<tg, 256, 0, c>>>(U, n, k0, nb, Linv);
+            float* P = U + (k0 + nb) * n + k0;         // the solved panel, rows k0+nb..n-1
+            const int64_t nb2 = imin64(kP, rest);      // width of the next panel
+            float* C = U + (k0 + nb) * n + k0 + nb;
+            if ((e = cudaEventRecord(la->panel_done, c)) != cudaSuccess) return e;
+            // the next block column also took the previous panel's rest update
+            if ((e = cudaStreamWaitEvent(c, la->rest_done, 0)) != cudaSuccess) return e;
+            e = launch_gemm<false, true, true>(C, n, P, n, P, n, rest, nb2, nb, -1.0f, c);
             if (e != cudaSuccess) return e;
+            if (rest > nb2) {
+                if ((e = cudaStreamWaitEvent(s, la->panel_done, 0)) != cudaSuccess) return e;
+                e = launch_gemm<false, true, true>(C + nb2 * n + nb2, n, P + nb2 * n, n, P + nb2 * n, n, rest - nb2,
+                                                   rest - nb2, nb, -1.0f, s);
+                if (e != cudaSuccess) return e;
+                if ((e = cudaEventRecord(la->rest_done, s)) != cudaSuccess) return e;
+            }
         }
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
+    if ((e = cudaEventRecord(la->crit_done, c)) != cudaSuccess) return e;          // join
+    if ((e = cudaStreamWaitEvent(s, la->crit_done, 0)) != cudaSuccess) return e;
+    lock.unlock();
     diag_d_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(U, n, D);
     flip_kernel<<<rg, 256, 0, s>>>(U, n);
     zero_diag_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(U, n);
