@@ -349,8 +349,10 @@ nvfp4_status nvfp4_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* 
  *   perm, U from nvfp4_ldlq_prepare (cols = n); status_dev optional: |= 8 if
  *   perm holds an index outside [0, cols) (the entry is then read as 0).
  *   workspace   device bytes, at least nvfp4_ldlq_workspace(rows, cols):
- *           rows*cols*10 + rows*1024 + cols*4 plus alignment.
- * Cost: rows*cols^2/2 fp32 multiply-adds; rows are independent.
+ *           rows*cols*10 + rows*2048 + cols*4 plus alignment.
+ * Cost: rows*cols^2/2 fp32 multiply-adds; rows are independent.  The column
+ * walk uses the high-priority stream described under nvfp4_ldlq_prepare (same
+ * first-call and concurrency rules).
  */
 size_t nvfp4_ldlq_workspace(int64_t rows, int64_t cols);
 nvfp4_status ldlq_quantize(const void* W, nvfp4_dtype dt, int64_t rows, int64_t cols, int block, const float* S,

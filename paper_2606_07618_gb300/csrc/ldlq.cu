@@ -664,16 +664,20 @@ cudaError_t launch_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* 
     return cudaGetLastError();
 }
 
-// Workspace: T and Wp [rows, n] f32, qb and sfp [rows, n] bytes, EpT [kLdlqPanel, rows] f32, inv [n].
+// Workspace: T and Wp [rows, n] f32, qb and sfp [rows, n] bytes, two EpT
+// [kLdlqPanel, rows] f32 (alternating between super-panels), inv [n].
 size_t ldlq_quantize_workspace(int64_t rows, int64_t n) {
     auto up = [](int64_t b) { return (b + 255) / 256 * 256; };
-    return (size_t)(2 * up(rows * n * 4) + 2 * up(rows * n) + up((int64_t)kLdlqPanel * rows * 4) + up(n * 4));
+    return (size_t)(2 * up(rows * n * 4) + 2 * up(rows * n) + 2 * up((int64_t)kLdlqPanel * rows * 4) + up(n * 4));
 }
 
 // Columns in super-panels of kLdlqPanel (256): each 64-column panel is walked by
 // panel_kernel and its errors update the rest of the super-panel at once (K = 64);
-// after the super-panel, one GEMM with K = 256 updates every later column, so the
-// targets are read and written once per 256 columns.
+// after the super-panel, GEMMs with K = 256 update every later column, so the
+// targets are read and written once per 256 columns.  Look-ahead: that update
+// is split into the next super-panel's columns, which run with its panel walks
+// on the high-priority stream, and the rest, which runs on `s` concurrently
+// with them; the super-panels' errors alternate between two EpT buffers.
 cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* ws, int sms, cudaStream_t s) {
     if (p.rows <= 0 || p.n <= 0) return cudaSuccess;
     auto up = [](int64_t b) { return (b + 255) / 256 * 256; };
@@ -683,8 +687,10 @@ cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* 
     p.Wp = reinterpret_cast<float*>(w + mat4);
     p.qb = reinterpret_cast<uint8_t*>(w + 2 * mat4);
     p.sfp = reinterpret_cast<uint8_t*>(w + 2 * mat4 + mat1);
-    float* EpT = reinterpret_cast<float*>(w + 2 * mat4 + 2 * mat1);
-    int32_t* inv = reinterpret_cast<int32_t*>(w + 2 * mat4 + 2 * mat1 + up((int64_t)kLdlqPanel * p.rows * 4));
+    const int64_t ep = up((int64_t)kLdlqPanel * p.rows * 4);
+    float* EpTs[2] = {reinterpret_cast<float*>(w + 2 * mat4 + 2 * mat1),
+                      reinterpret_cast<float*>(w + 2 * mat4 + 2 * mat1 + ep)};
+    int32_t* inv = reinterpret_cast<int32_t*>(w + 2 * mat4 + 2 * mat1 + 2 * ep);
     cudaError_t e = cudaMemsetAsync(inv, 0, (size_t)p.n * 4, s);
     if (e != cudaSuccess) return e;
     invperm_kernel<<<(unsigned)((p.n + 255) / 256), 256, 0, s>>>(p.perm, p.n, inv, p.status);
@@ -707,31 +713,56 @@ cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* 
         if (dev >= 0 && dev < 64) attr_set[dev].store(true, std::memory_order_release);
     }
     const unsigned pg = (unsigned)imin64((p.rows + kPanelRows - 1) / kPanelRows, (int64_t)sms * 16);
-    for (int64_t s0 = 0; s0 < p.n; s0 += kLdlqPanel) {
+    LookAhead* la = nullptr;
+    std::unique_lock<std::mutex> lock;
+    e = lookahead_for_current_device(&la, &lock);
+    if (e != cudaSuccess) return e;
+    cudaStream_t c = la->crit;
+    if ((e = cudaEventRecord(la->fork, s)) != cudaSuccess) return e;
+    if ((e = cudaStreamWaitEvent(c, la->fork, 0)) != cudaSuccess) return e;
+    int sp = 0;
+    for (int64_t s0 = 0; s0 < p.n; s0 += kLdlqPanel, sp++) {
         const int64_t span = imin64(kLdlqPanel, p.n - s0);
+        float* EpT = EpTs[sp & 1];
         for (int64_t k0 = s0; k0 < s0 + span; k0 += kP) {
             const int P = (int)imin64(kP, s0 + span - k0);
             float* Ek = EpT + (k0 - s0) * p.rows;
             if (dtype == 0)
-                panel_kernel<0><<<pg, kPanelThreads, kPanelSmem, s>>>(p, k0, P, Ek);
+                panel_kernel<0><<<pg, kPanelThreads, kPanelSmem, c>>>(p, k0, P, Ek);
             else
-                panel_kernel<1><<<pg, kPanelThreads, kPanelSmem, s>>>(p, k0, P, Ek);
+                panel_kernel<1><<<pg, kPanelThreads, kPanelSmem, c>>>(p, k0, P, Ek);
             e = cudaGetLastError();
             if (e != cudaSuccess) return e;
             const int64_t rest_in = s0 + span - (k0 + P);
             if (rest_in > 0) {
                 e = launch_gemm<true, false, false>(p.T + k0 + P, p.n, Ek, p.rows, p.U + k0 * p.n + k0 + P, p.n,
-                                                    p.rows, rest_in, P, 1.0f, s);
+                                                    p.rows, rest_in, P, 1.0f, c);
                 if (e != cudaSuccess) return e;
             }
         }
         const int64_t rest = p.n - (s0 + span);
         if (rest > 0) {
+            const int64_t next = imin64(kLdlqPanel, rest);
+            if ((e = cudaEventRecord(la->panel_done, c)) != cudaSuccess) return e;
+            // the next super-panel's columns also took the previous rest update, and
+            // that update read the EpT buffer the next super-panel overwrites
+            if ((e = cudaStreamWaitEvent(c, la->rest_done, 0)) != cudaSuccess) return e;
             e = launch_gemm<true, false, false>(p.T + s0 + span, p.n, EpT, p.rows, p.U + s0 * p.n + s0 + span, p.n,
-                                                p.rows, rest, (int)span, 1.0f, s);
+                                                p.rows, next, (int)span, 1.0f, c);
             if (e != cudaSuccess) return e;
+            if (rest > next) {
+                if ((e = cudaStreamWaitEvent(s, la->panel_done, 0)) != cudaSuccess) return e;
+                e = launch_gemm<true, false, false>(p.T + s0 + span + next, p.n, EpT, p.rows,
+                                                    p.U + s0 * p.n + s0 + span + next, p.n, p.rows, rest - next,
+                                                    (int)span, 1.0f, s);
+                if (e != cudaSuccess) return e;
+                if ((e = cudaEventRecord(la->rest_done, s)) != cudaSuccess) return e;
+            }
         }
     }
+    if ((e = cudaEventRecord(la->crit_done, c)) != cudaSuccess) return e;          // join
+    if ((e = cudaStreamWaitEvent(s, la->crit_done, 0)) != cudaSuccess) return e;
+    lock.unlock();
     pack_kernel<<<rg, 256, 0, s>>>(p.qb, inv, p.rows, p.n, codes, p.status);
     return cudaGetLastError();
 }
