@@ -629,6 +629,7 @@ cudaError_t launch_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* 
     cudaStream_t c = la->crit;
     if ((e = cudaEventRecord(la->fork, s)) != cudaSuccess) return e;
     if ((e = cudaStreamWaitEvent(c, la->fork, 0)) != cudaSuccess) return e;
+    bool have_rest = false;              // rest_done recorded by this call (waits stay inside a capture)
     for (int64_t k0 = 0; k0 < n; k0 += kP) {
         const int nb = (int)imin64(kP, n - k0);
         potrf_kernel<<<1, 256, 0, c>>>(U, n, k0, nb, Linv, status);
@@ -641,7 +642,7 @@ cudaError_t launch_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* 
             float* C = U + (k0 + nb) * n + k0 + nb;
             if ((e = cudaEventRecord(la->panel_done, c)) != cudaSuccess) return e;
             // the next block column also took the previous panel's rest update
-            if ((e = cudaStreamWaitEvent(c, la->rest_done, 0)) != cudaSuccess) return e;
+            if (have_rest && (e = cudaStreamWaitEvent(c, la->rest_done, 0)) != cudaSuccess) return e;
             e = launch_gemm<false, true, true>(C, n, P, n, P, n, rest, nb2, nb, -1.0f, c);
             if (e != cudaSuccess) return e;
             if (rest > nb2) {
@@ -650,6 +651,7 @@ cudaError_t launch_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* 
                                                    rest - nb2, nb, -1.0f, s);
                 if (e != cudaSuccess) return e;
                 if ((e = cudaEventRecord(la->rest_done, s)) != cudaSuccess) return e;
+                have_rest = true;
             }
         }
         e = cudaGetLastError();
@@ -720,6 +722,7 @@ cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* 
     cudaStream_t c = la->crit;
     if ((e = cudaEventRecord(la->fork, s)) != cudaSuccess) return e;
     if ((e = cudaStreamWaitEvent(c, la->fork, 0)) != cudaSuccess) return e;
+    bool have_rest = false;              // rest_done recorded by this call (waits stay inside a capture)
     int sp = 0;
     for (int64_t s0 = 0; s0 < p.n; s0 += kLdlqPanel, sp++) {
         const int64_t span = imin64(kLdlqPanel, p.n - s0);
@@ -746,7 +749,7 @@ cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* 
             if ((e = cudaEventRecord(la->panel_done, c)) != cudaSuccess) return e;
             // the next super-panel's columns also took the previous rest update, and
             // that update read the EpT buffer the next super-panel overwrites
-            if ((e = cudaStreamWaitEvent(c, la->rest_done, 0)) != cudaSuccess) return e;
+            if (have_rest && (e = cudaStreamWaitEvent(c, la->rest_done, 0)) != cudaSuccess) return e;
             e = launch_gemm<true, false, false>(p.T + s0 + span, p.n, EpT, p.rows, p.U + s0 * p.n + s0 + span, p.n,
                                                 p.rows, next, (int)span, 1.0f, c);
             if (e != cudaSuccess) return e;
@@ -757,6 +760,7 @@ cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* 
                                                     (int)span, 1.0f, s);
                 if (e != cudaSuccess) return e;
                 if ((e = cudaEventRecord(la->rest_done, s)) != cudaSuccess) return e;
+                have_rest = true;
             }
         }
     }

@@ -204,3 +204,40 @@ def test_failures_are_reported_not_faulted(B):
     bad_perm[3] = n + 5
     codes, st3 = quantize(B, W, 0.001, np.full((4, n // 16), 60, np.uint8), bad_perm, U)
     assert st3 & 8
+
+
+def test_prepare_and_quantize_captured_in_cuda_graph(B):
+    """Both calls (their look-ahead forks a high-priority stream and joins it
+    back) captured in one CUDA graph and replayed: the eager results, bit for
+    bit."""
+    rows, n = 64, 320
+    W64, H = rand_problem(rows, n, 77)
+    Wt = torch.from_numpy(W64.astype(np.float32)).to(DEV)
+    H = H.astype(np.float32).astype(np.float64)
+    S, sf = fixed_scales(W64, H)
+    perm, U, D, st = prepare(B, H)                         # eager (also the first call on the device)
+    codes, st1 = quantize(B, Wt, S, sf, perm, U)
+    assert st == 0 and st1 == 0
+    Hd = torch.as_tensor(H, dtype=torch.float32).to(DEV)
+    perm2 = torch.empty(n, dtype=torch.int32, device=DEV)
+    U2 = torch.empty(n, n, dtype=torch.float32, device=DEV)
+    D2 = torch.empty(n, dtype=torch.float32, device=DEV)
+    codes2 = torch.empty(rows, n // 2, dtype=torch.uint8, device=DEV)
+    st2 = torch.zeros(1, dtype=torch.int32, device=DEV)
+    wsp = torch.empty(B.nvfp4_ldlq_prepare_workspace(n), dtype=torch.uint8, device=DEV)
+    wsq = torch.empty(B.nvfp4_ldlq_workspace(rows, n), dtype=torch.uint8, device=DEV)
+    Sd = torch.tensor([S], dtype=torch.float32, device=DEV)
+    sfd = torch.as_tensor(np.ascontiguousarray(sf), dtype=torch.uint8).to(DEV)
+    s = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        B.nvfp4_ldlq_prepare(Hd, 0.01, perm2, U2, D2, st2, wsp, stream=s)
+        B.ldlq_quantize(Wt, 16, Sd, sfd, perm2, U2, codes2, st2, wsq, stream=s)
+    for _ in range(2):
+        codes2.zero_()
+        g.replay()
+        torch.cuda.synchronize()
+        assert st2.item() == 0
+        assert torch.equal(perm2, perm) and torch.equal(U2, U) and torch.equal(D2, D)
+        assert np.array_equal(codes2.cpu().numpy(), codes)
