@@ -443,8 +443,14 @@ __global__ void __launch_bounds__(256) gather_w_kernel(LdlqParams p) {
 // c <= s and past the panel).  Splitting the 64-wide update shortens the
 // sequential chain per column four-fold.  The CTA's 32 rows of original weights
 // and scale codes are staged in shared memory with coalesced loads first.
+#ifndef NVFP4_PANEL_TPR
+#define NVFP4_PANEL_TPR 8
+#endif
 constexpr int kPanelThreads = 128;
-constexpr int kPanelRows = kPanelThreads / 4;
+constexpr int kPanelTpr = NVFP4_PANEL_TPR;          // threads per row
+constexpr int kPanelTargets = kP / kPanelTpr;       // targets per thread
+constexpr int kPanelRows = kPanelThreads / kPanelTpr;
+static_assert(kPanelTargets % 4 == 0 && 16 % kPanelTargets == 0, "a thread's targets are whole float4s within a block");
 constexpr int kPanelSmem = (kP * kP + 128 + kPanelRows * (kP + 1)) * 4 + kPanelRows * (kP + 4);
 
 template <int DT>
@@ -465,8 +471,8 @@ __global__ void __launch_bounds__(kPanelThreads) panel_kernel(LdlqParams p, int6
     const bool usable = (S > 0.0f) && isfinite(S) && isfinite(Einv);
     const float E = usable ? Einv : 1.0f;
     const int lane = threadIdx.x & 31;
-    const int kq = threadIdx.x & 3;                   // this thread's quarter of the columns
-    const int rr = threadIdx.x >> 2;                  // row within the CTA's block
+    const int kq = threadIdx.x % kPanelTpr;           // this thread's share of the columns
+    const int rr = threadIdx.x / kPanelTpr;           // row within the CTA's block
     for (int64_t rb = (int64_t)blockIdx.x * kPanelRows; rb < p.rows; rb += (int64_t)gridDim.x * kPanelRows) {
         __syncthreads();                              // previous row block done with wsm/csm
         {
@@ -491,11 +497,11 @@ __global__ void __launch_bounds__(kPanelThreads) panel_kernel(LdlqParams p, int6
         }
         __syncthreads();
         const int64_t r = rb + rr;
-        const bool active = r < p.rows;               // a whole quad shares r
-        const int c0 = 16 * kq;
-        float t[16];
+        const bool active = r < p.rows;               // a row's threads share r
+        const int c0 = kPanelTargets * kq;
+        float t[kPanelTargets];
 #pragma unroll
-        for (int g = 0; g < 4; g++) {
+        for (int g = 0; g < kPanelTargets / 4; g++) {
             const float4 v = (active && c0 + 4 * g < P) ? *reinterpret_cast<const float4*>(p.T + r * p.n + k0 + c0 + 4 * g)
                                                         : make_float4(0, 0, 0, 0);
             t[4 * g] = v.x;
@@ -503,14 +509,14 @@ __global__ void __launch_bounds__(kPanelThreads) panel_kernel(LdlqParams p, int6
             t[4 * g + 2] = v.z;
             t[4 * g + 3] = v.w;
         }
-        uint32_t packed[4] = {0, 0, 0, 0};
+        uint32_t packed[kPanelTargets / 4] = {};
 #pragma unroll 1
-        for (int kb = 0; kb < P / 16; kb++) {          // the quarter whose columns are walked now
+        for (int kb = 0; kb < P / kPanelTargets; kb++) {   // the share whose columns are walked now
             const bool owner = kq == kb;
-            const int src = (lane & ~3) | kb;
+            const int src = (lane & ~(kPanelTpr - 1)) | kb;
 #pragma unroll
-            for (int j = 0; j < 16; j++) {
-                const int s = 16 * kb + j;
+            for (int j = 0; j < kPanelTargets; j++) {
+                const int s = kPanelTargets * kb + j;
                 float e = 0.0f;
                 if (owner && active) {
                     const int cs = csm[rr][s];
@@ -540,7 +546,7 @@ __global__ void __launch_bounds__(kPanelThreads) panel_kernel(LdlqParams p, int6
                 e = __shfl_sync(0xffffffffu, e, src);
                 const float* us = &up[s][c0];
 #pragma unroll
-                for (int g = 0; g < 4; g++) {
+                for (int g = 0; g < kPanelTargets / 4; g++) {
                     const float4 u = *reinterpret_cast<const float4*>(us + 4 * g);
                     t[4 * g + 0] = __fmaf_rn(e, u.x, t[4 * g + 0]);
                     t[4 * g + 1] = __fmaf_rn(e, u.y, t[4 * g + 1]);
@@ -549,8 +555,15 @@ __global__ void __launch_bounds__(kPanelThreads) panel_kernel(LdlqParams p, int6
                 }
             }
         }
-        if (active && c0 < P)
-            *reinterpret_cast<uint4*>(p.qb + r * p.n + k0 + c0) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+        if (active && c0 < P) {
+            uint8_t* q = p.qb + r * p.n + k0 + c0;    // one byte per column: kPanelTargets bytes
+            if constexpr (kPanelTargets == 16)
+                *reinterpret_cast<uint4*>(q) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+            else if constexpr (kPanelTargets == 8)
+                *reinterpret_cast<uint2*>(q) = make_uint2(packed[0], packed[1]);
+            else
+                *reinterpret_cast<uint32_t*>(q) = packed[0];
+        }
     }
 }
 
