@@ -69,7 +69,7 @@ typedef enum { NVFP4_SF_LINEAR = 1, NVFP4_SF_SWIZZLED = 2 } nvfp4_sf_layout;
  * beats s/2, which is code c - 8 and stays in the window; 3.5 v_c is exact in
  * fp32; below code 16 half a scale need not be a code), and for MSE with block
  * 16 the lower end is the
- * per-mantissa bound of Table 3 (I0 - 2, or I0 - 3 for mantissas 000 and 111;
+ * per-mantissa bound of Table 2 (I0 - 2, or I0 - 3 for mantissas 000 and 111;
  * applied for I0 in 16..120, where the ceiling stays normal and Lemma 4.3's
  * 11/7 s <= 448 holds).  A warp runs as many candidates as its widest block. */
 #define NVFP4_WINDOW_TIGHT (INT_MIN + 1)

@@ -22,7 +22,7 @@ struct QuantParams {
     int need_rowcol;         // swizzled scales or weights need (row, block column)
     FastDiv kb_div;          // divides a 32-bit block index by kb
     int win_lo, win_hi;
-    int tight;               // per-block window: bit 0 Lemma 4.1 upper cut, bit 1 Table 3 lower (MSE, block 16)
+    int tight;               // per-block window: bit 0 Lemma 4.1 upper cut, bit 1 Table 2 lower (MSE, block 16)
     uint8_t* codes;
     uint8_t* sf_linear;
     uint8_t* sf_swizzled;

@@ -375,7 +375,7 @@ __global__ void __launch_bounds__(256, NVFP4_QMINB) quantize_kernel(QuantParams 
             } else {
                 int lo_off = p.win_lo;
                 if ((p.tight & 2) && I0 >= 16 && I0 <= 120) {
-                    const int b = I0 & 7;                       // Table 3: ceil(4/5 s) is 2 or 3 codes down
+                    const int b = I0 & 7;                       // Table 2: ceil(4/5 s) is 2 or 3 codes down
                     lo_off = (b == 0 || b == 7) ? -3 : -2;
                 }
                 const int clo = min(max(I0 + lo_off, 1), 126);

@@ -5,7 +5,7 @@ dropping candidates the paper proves useless, block by block:
 * upper end: every code c >= 16 with 3.5 v_c > max|y| goes (Lemma 4.1: such a
   scale never beats half of it, which is code c - 8 and stays in the window;
   below 16 half a scale need not be a code -- subnormal code 3 has no half);
-* lower end, MSE with 16-element blocks: the per-mantissa bound of Table 3 /
+* lower end, MSE with 16-element blocks: the per-mantissa bound of Table 2 /
   Lemma 4.3, I0 - delta(b) with delta from the exact rational table in
   oracle/bounds.py (not from the kernel's constants), for I0 in 16..120.
 Checked on the oracle's float64 candidate losses: the argmin over each block's
@@ -109,7 +109,7 @@ def test_tight_window_prunes_and_planted_mistakes_are_caught():
     live = m2 > 0
     clo2, chi2 = tight_windows(m2, I02, oracle.MSE, 16, cut_from=1)
     assert not np.array_equal(tight_choice(ref2, clo2, chi2)[live], ref2["sf"].reshape(-1)[live].astype(np.int64))
-    # the lower end is tightened where it applies (Table 3 itself is pinned
+    # the lower end is tightened where it applies (Table 2 itself is pinned
     # against the paper's printed table in test_oracle_bounds.py; no sampled block
     # sits at it, so a bound one code too high cannot be caught by results)
     rng16 = (I0 >= 16) & (I0 <= 120)
