@@ -612,6 +612,8 @@ def run_table7(args):
     from paper_2606_07618_gb300 import workloads as W
     dev = "cuda"
     win = (B.NVFP4_WINDOW_DEFAULT, B.NVFP4_WINDOW_DEFAULT)
+    l2 = torch.cuda.get_device_properties(torch.cuda.current_device()).L2_cache_size
+    flush = torch.empty(2 * l2 // 4, dtype=torch.float32, device=dev)
     rows = []
     for b in (128, 256, 512, 1024, 2048, 4096, 8192, 16384, 32768):
         t = W.workload(f"table7-{b}").tensors[0]
@@ -664,6 +666,21 @@ def run_table7(args):
             e.record()
             torch.cuda.synchronize()
             res[kind + "_ms"] = round(a.elapsed_time(e) / reps, 4)
+        # Cold L2: before every timed call a buffer of twice the L2 size is
+        # rewritten (the call's own launch is already queued when the flush ends,
+        # so the events see the device time of the call with its inputs in HBM).
+        for kind in ("absmax", "mse", "wmse"):
+            f = op(kind)
+            tot = 0.0
+            for _ in range(20):
+                flush.add_(1.0)
+                a, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record()
+                f()
+                e.record()
+                torch.cuda.synchronize()
+                tot += a.elapsed_time(e)
+            res[kind + "_l2flush_ms"] = round(tot / 20, 4)
         # The same calls captured once in a CUDA graph and replayed: the library
         # never allocates or synchronises, so a caller can remove the per-call
         # host cost this way; what remains is the device time per call.
