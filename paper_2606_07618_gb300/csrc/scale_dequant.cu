@@ -6,6 +6,9 @@
 // workspace, then a single CTA folds the partials and writes S on the device.
 // No atomics and no zero-initialised state, so back-to-back calls on one
 // workspace need nothing in between.  Max is exact, so the order is free.
+// The folding CTA is a programmatic dependent launch: it is scheduled while
+// the partial grid drains and waits (griddepcontrol.wait) for that grid's
+// writes, which takes its launch latency off the critical path.
 #include <cuda_bf16.h>
 
 #include "nvfp4_device.cuh"
@@ -19,7 +22,7 @@ __device__ __forceinline__ void amax_acc(float v, float& m, int& bad) {
 }
 
 template <int DT>
-__global__ void __launch_bounds__(256) amax_partial_kernel(const void* x, int64_t n, float* part_max,
+__global__ void __launch_bounds__(512) amax_partial_kernel(const void* x, int64_t n, float* part_max,
                                                            int* part_bad) {
     constexpr int PER = DT == 0 ? 8 : 4;      // elements per 16-byte vector
     const int64_t nvec = n / PER;
@@ -40,16 +43,14 @@ __global__ void __launch_bounds__(256) amax_partial_kernel(const void* x, int64_
         }
     };
     int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    // four independent 16-byte loads in flight per thread
-    for (; i + 3 * stride < nvec; i += 4 * stride) {
+    // two independent 16-byte loads in flight per thread; with 2048 threads
+    // per SM that keeps ~10 MB in flight across the GPU
+    for (; i + stride < nvec; i += 2 * stride) {
         const uint4 u0 = ld_stream16(xv + i), u1 = ld_stream16(xv + i + stride);
-        const uint4 u2 = ld_stream16(xv + i + 2 * stride), u3 = ld_stream16(xv + i + 3 * stride);
         fold(u0);
         fold(u1);
-        fold(u2);
-        fold(u3);
     }
-    for (; i < nvec; i += stride) fold(ld_stream16(xv + i));
+    if (i < nvec) fold(ld_stream16(xv + i));
     // tail elements (n not a multiple of the vector width)
     if (blockIdx.x == 0 && threadIdx.x < (int)(n - nvec * PER)) {
         const int64_t i = nvec * PER + threadIdx.x;
@@ -57,11 +58,13 @@ __global__ void __launch_bounds__(256) amax_partial_kernel(const void* x, int64_
                           : static_cast<const float*>(x)[i];
         amax_acc(v, m, bad);
     }
+    // every load of this CTA has returned: let the folding kernel be scheduled
+    grid_launch_dependents();
     // non-negative floats order like their bit patterns
     uint32_t mb = __reduce_max_sync(0xffffffffu, __float_as_uint(m));
     int anybad = __reduce_or_sync(0xffffffffu, (unsigned)bad);
-    __shared__ uint32_t sm[8];
-    __shared__ int sb[8];
+    __shared__ uint32_t sm[16];
+    __shared__ int sb[16];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) {
         sm[warp] = mb;
@@ -82,6 +85,9 @@ __global__ void __launch_bounds__(256) amax_partial_kernel(const void* x, int64_
 
 __global__ void __launch_bounds__(256) amax_final_kernel(const float* part_max, const int* part_bad, int nparts,
                                                          float fp8_div, float* S_out, int* status_dev) {
+    // launched as a programmatic dependent of amax_partial_kernel: wait until
+    // that grid has finished and its partials are visible (a no-op otherwise)
+    grid_dependency_wait();
     uint32_t v = 0u;
     int b = 0;
     for (int i = threadIdx.x; i < nparts; i += blockDim.x) {
@@ -111,39 +117,54 @@ __global__ void __launch_bounds__(256) amax_final_kernel(const float* part_max, 
     }
 }
 
+// The folding CTA, allowed to start before amax_partial_kernel has drained.
+static cudaError_t launch_final(const float* part_max, const int* part_bad, int nparts, float fp8_div,
+                                float* S_out, int* status_dev, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(1);
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, amax_final_kernel, part_max, part_bad, nparts, fp8_div, S_out, status_dev);
+}
+
+static cudaError_t launch_partial(const void* x, int dtype, int64_t n, float* part_max, int* part_bad, int grid,
+                                  int threads, cudaStream_t s) {
+    if (dtype == 0)
+        amax_partial_kernel<0><<<grid, threads, 0, s>>>(x, n, part_max, part_bad);
+    else
+        amax_partial_kernel<1><<<grid, threads, 0, s>>>(x, n, part_max, part_bad);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_global_scale(const void* x, int dtype, int64_t n, float fp8_div, float* S_out,
                                 int* status_dev, void* ws, int sms, cudaStream_t s) {
     float* part_max = static_cast<float*>(ws);
     int* part_bad = reinterpret_cast<int*>(part_max + kAmaxParts);
-    // 128-thread CTAs (~4K registers each) so the reduction can share SMs with
-    // an ALU-bound sweep running on another stream.
-    constexpr int kThreads = 128;
+    // 512-thread CTAs, 4 per SM, two loads in flight each: measured fastest of
+    // 128/256/512 threads x 1/2/4/8 loads and of 32-byte loads on GB300
+    constexpr int kThreads = 512;
     const int per = dtype == 0 ? 8 : 4;
     const int64_t nvec = n / per;
-    int64_t grid = (nvec + kThreads * 4 - 1) / (kThreads * 4);
-    if (grid > (int64_t)sms * 6) grid = (int64_t)sms * 6;
+    int64_t grid = (nvec + kThreads * 2 - 1) / (kThreads * 2);
+    if (grid > (int64_t)sms * 4) grid = (int64_t)sms * 4;
     if (grid > kAmaxParts) grid = kAmaxParts;
     if (grid < 1) grid = 1;
-    if (dtype == 0)
-        amax_partial_kernel<0><<<(int)grid, kThreads, 0, s>>>(x, n, part_max, part_bad);
-    else
-        amax_partial_kernel<1><<<(int)grid, kThreads, 0, s>>>(x, n, part_max, part_bad);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_partial(x, dtype, n, part_max, part_bad, (int)grid, kThreads, s);
     if (e != cudaSuccess) return e;
-    amax_final_kernel<<<1, 256, 0, s>>>(part_max, part_bad, (int)grid, fp8_div, S_out, status_dev);
-    return cudaGetLastError();
+    return launch_final(part_max, part_bad, (int)grid, fp8_div, S_out, status_dev, s);
 }
 
 cudaError_t launch_global_scale_parts(const void* x, int dtype, int64_t n, float fp8_div, float* S_out,
                                       int* status_dev, float* part_max, int* part_bad, int grid, cudaStream_t s) {
-    if (dtype == 0)
-        amax_partial_kernel<0><<<grid, 256, 0, s>>>(x, n, part_max, part_bad);
-    else
-        amax_partial_kernel<1><<<grid, 256, 0, s>>>(x, n, part_max, part_bad);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_partial(x, dtype, n, part_max, part_bad, grid, 256, s);
     if (e != cudaSuccess) return e;
-    amax_final_kernel<<<1, 256, 0, s>>>(part_max, part_bad, grid, fp8_div, S_out, status_dev);
-    return cudaGetLastError();
+    return launch_final(part_max, part_bad, grid, fp8_div, S_out, status_dev, s);
 }
 
 // ---------------------------------------------------------------------------
