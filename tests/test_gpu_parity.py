@@ -257,12 +257,13 @@ def test_dynamic_scale_on_side_stream_and_determinism(B):
 # --------------------------------------------------------------------------- dequantisation
 @pytest.mark.parametrize("block", [16, 32, 64])
 @pytest.mark.parametrize("out_dtype", [torch.float32, torch.bfloat16])
-def test_dequantize_bit_exact(B, block, out_dtype):
+@pytest.mark.parametrize("S_val", [0.0371, 1e-39, 3e36])     # ordinary; subnormal S; products past fp32/bf16 max
+def test_dequantize_bit_exact(B, block, out_dtype, S_val):
     rows, cols = 131, 256
     g = np.random.default_rng(block)
     codes = g.integers(0, 256, (rows, cols // 2), dtype=np.uint8)
     sf = g.integers(0, 127, (rows, cols // block), dtype=np.uint8)
-    S = np.float32(0.0371)
+    S = np.float32(S_val)
     Sd = torch.tensor([S], device=DEV)
     layouts = [(1, sf)] + ([(2, oracle.swizzle_scales(sf))] if block == 16 else [])
     for layout, sfl in layouts:
