@@ -277,11 +277,17 @@ __device__ __forceinline__ bool dynamic_scale(const QuantParams& p, float& S_out
 
 // FIX = 1: default window (fixed length, unrolled, poison-padded table).
 // DYN = 1: the global scale is computed in this launch (see dynamic_scale).
-// AbsMax on bf16 is held to 64 registers for 4 CTAs per SM: it is issue- and
-// latency-bound, not register-bound (0.0677 -> 0.0636 ms at 16384 x 8192; the
-// fp32-input forms would spill at that bound).
+// On bf16 input, AbsMax is held to 64 registers (4 CTAs per SM) and 4/6 to 80
+// (3 CTAs per SM): both are issue- and latency-bound, not register-bound (AbsMax
+// 0.0677 -> 0.0636 ms, 4/6 WMSE 0.120 -> 0.115 ms at 16384 x 8192; the
+// fp32-input forms would spill, and the ScaleSweep sweeps run slower, at such bounds).
+template <int METHOD, int DT>
+constexpr int quantize_min_blocks() {
+    return DT != 0 ? NVFP4_QMINB : (METHOD == 1 ? 4 : (METHOD == 2 ? 3 : NVFP4_QMINB));
+}
+
 template <int DT, int METHOD, int OBJ, int BLOCK, int FIX, int DYN>
-__global__ void __launch_bounds__(256, (METHOD == 1 && DT == 0) ? 4 : NVFP4_QMINB) quantize_kernel(QuantParams p) {
+__global__ void __launch_bounds__(256, quantize_min_blocks<METHOD, DT>()) quantize_kernel(QuantParams p) {
     constexpr int SEGS = BLOCK / 16;
     constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
     constexpr int FIX_K = 7 - FIX_LO + 1;
