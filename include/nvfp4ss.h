@@ -91,7 +91,9 @@ size_t nvfp4_global_scale_workspace(int64_t n);
  *              (NaNs are ignored by the max, an inf makes S = inf).
  *   workspace  device scratch of nvfp4_global_scale_workspace(n) bytes,
  *              16-byte aligned; its contents need no initialisation.
- * n == 0 writes S = 0.  Two kernel launches on `stream`.
+ * n == 0 writes S = 0.  Two kernel launches on `stream`, the second a
+ * programmatic dependent launch of the first (scheduled while the first drains,
+ * ordered after its writes); both can be captured in a CUDA graph.
  */
 nvfp4_status nvfp4_global_scale(const void* x, nvfp4_dtype dt, int64_t n, float fp8_div, float* S_out,
                                 int* status_dev, void* workspace, size_t ws_bytes, void* stream);
