@@ -162,3 +162,42 @@ def test_group_validation_without_gpu(L):
     assert st_test(which=2) == 1
     assert st_test(status=None) == 1                 # the status word is how the timeout is seen
     assert st_test(rows=0) == 1
+
+
+def test_header_constants_and_struct_layout_match_the_binding(tmp_path):
+    """Compile a C probe against include/nvfp4ss.h with the host C compiler and
+    compare the enum values, the window and group constants and the layout of
+    nvfp4_group_tensor with what the Python binding passes through ctypes."""
+    import shutil
+    import subprocess
+    from paper_2606_07618_gb300 import binding as B
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no host C compiler")
+    src = tmp_path / "probe.c"
+    src.write_text(r'''
+#include <stdio.h>
+#include "nvfp4ss.h"
+#define F(name) printf(#name " %zu %zu\n", offsetof(nvfp4_group_tensor, name), sizeof(((nvfp4_group_tensor*)0)->name))
+int main(void) {
+    printf("size %zu\n", sizeof(nvfp4_group_tensor));
+    F(x); F(rows); F(cols); F(w); F(w_row_stride); F(codes); F(sf_linear); F(sf_swizzled);
+    printf("NVFP4_IN_BF16 %d\nNVFP4_IN_F32 %d\nNVFP4_OBJ_MSE %d\nNVFP4_OBJ_WMSE %d\n", NVFP4_IN_BF16, NVFP4_IN_F32,
+           NVFP4_OBJ_MSE, NVFP4_OBJ_WMSE);
+    printf("NVFP4_SF_LINEAR %d\nNVFP4_SF_SWIZZLED %d\n", NVFP4_SF_LINEAR, NVFP4_SF_SWIZZLED);
+    printf("NVFP4_WINDOW_DEFAULT %d\nNVFP4_WINDOW_TIGHT %d\nNVFP4_GROUP_MAX %d\n", NVFP4_WINDOW_DEFAULT,
+           NVFP4_WINDOW_TIGHT, NVFP4_GROUP_MAX);
+    return 0;
+}
+''')
+    exe = tmp_path / "probe"
+    subprocess.run([cc, "-std=c99", "-I", os.path.dirname(HEADER), str(src), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split("\n")
+    vals = {ln.split()[0]: [int(v) for v in ln.split()[1:]] for ln in out if ln.strip()}
+    assert vals["size"] == [ctypes.sizeof(B.GroupTensor)]
+    for name, _ in B.GroupTensor._fields_:
+        f = getattr(B.GroupTensor, name)
+        assert vals[name] == [f.offset, f.size], name
+    for name in ("NVFP4_IN_BF16", "NVFP4_IN_F32", "NVFP4_OBJ_MSE", "NVFP4_OBJ_WMSE", "NVFP4_SF_LINEAR",
+                 "NVFP4_SF_SWIZZLED", "NVFP4_WINDOW_DEFAULT", "NVFP4_WINDOW_TIGHT", "NVFP4_GROUP_MAX"):
+        assert vals[name] == [getattr(B, name)], name
