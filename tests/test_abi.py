@@ -201,3 +201,39 @@ int main(void) {
     for name in ("NVFP4_IN_BF16", "NVFP4_IN_F32", "NVFP4_OBJ_MSE", "NVFP4_OBJ_WMSE", "NVFP4_SF_LINEAR",
                  "NVFP4_SF_SWIZZLED", "NVFP4_WINDOW_DEFAULT", "NVFP4_WINDOW_TIGHT", "NVFP4_GROUP_MAX"):
         assert vals[name] == [getattr(B, name)], name
+
+
+def _declared_signatures():
+    src = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    sigs = {}
+    for m in re.finditer(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\**\s+([a-z0-9_]+)\s*\(([^)]*)\)\s*;", src, re.M):
+        params = [p.strip() for p in m.group(2).replace("\n", " ").split(",") if p.strip()]
+        if params == ["void"]:
+            params = []
+        sigs[m.group(1)] = params
+    return sigs
+
+
+def _ctype_of(param):
+    from paper_2606_07618_gb300 import binding as B
+    decl = param.rsplit(None, 1)[0] if not param.endswith("*") else param
+    if "*" in param:
+        return ctypes.POINTER(B.GroupTensor) if "nvfp4_group_tensor" in param else ctypes.c_void_p
+    t = decl.replace("const", "").strip()
+    return {"int": ctypes.c_int, "int64_t": ctypes.c_int64, "float": ctypes.c_float, "size_t": ctypes.c_size_t,
+            "nvfp4_dtype": ctypes.c_int, "nvfp4_objective": ctypes.c_int, "nvfp4_sf_layout": ctypes.c_int,
+            "nvfp4_status": ctypes.c_int}[t]
+
+
+def test_binding_argtypes_match_the_header(L):
+    """Every entry point's ctypes argument list has the header's arity and C types
+    (pointers as void*, enums as int), so no argument is passed at the wrong width."""
+    sigs = _declared_signatures()
+    assert sorted(sigs) == declared_functions()
+    for name, params in sigs.items():
+        got = getattr(L, name).argtypes
+        assert got is not None, name
+        want = [_ctype_of(p) for p in params]
+        assert len(got) == len(want), name
+        for i, (g, w) in enumerate(zip(got, want)):
+            assert g == w, (name, i, params[i])
