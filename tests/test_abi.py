@@ -225,11 +225,21 @@ def _ctype_of(param):
             "nvfp4_status": ctypes.c_int}[t]
 
 
+def _declared_return_types():
+    src = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    return {m.group(2): m.group(1).strip() for m in
+            re.finditer(r"^\s*((?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\**)\s+([a-z0-9_]+)\s*\(", src, re.M)}
+
+
 def test_binding_argtypes_match_the_header(L):
     """Every entry point's ctypes argument list has the header's arity and C types
-    (pointers as void*, enums as int), so no argument is passed at the wrong width."""
+    (pointers as void*, enums as int), so no argument is passed at the wrong width,
+    and its result type is the header's (status as int, sizes as size_t)."""
     sigs = _declared_signatures()
     assert sorted(sigs) == declared_functions()
+    ret = {"nvfp4_status": ctypes.c_int, "size_t": ctypes.c_size_t, "const char*": ctypes.c_char_p}
+    for name, rt in _declared_return_types().items():
+        assert getattr(L, name).restype == ret[rt.replace(" *", "*")], (name, rt)
     for name, params in sigs.items():
         got = getattr(L, name).argtypes
         assert got is not None, name
