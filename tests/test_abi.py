@@ -247,3 +247,17 @@ def test_binding_argtypes_match_the_header(L):
         assert len(got) == len(want), name
         for i, (g, w) in enumerate(zip(got, want)):
             assert g == w, (name, i, params[i])
+
+
+def test_build_covers_every_source_for_sm_103a():
+    """Every CUDA translation unit in csrc/ is compiled, for sm_103a only, and
+    every header it includes counts towards the rebuild check."""
+    from paper_2606_07618_gb300 import build as Bd
+    cu = sorted(f for f in os.listdir(Bd.CSRC) if f.endswith(".cu"))
+    assert sorted(Bd.SOURCES) == cu
+    assert Bd.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
+    flags = Bd._flags(False)
+    assert "-O3" in flags and "-lineinfo" in flags
+    inputs = set(os.path.basename(f) for f in Bd._inputs())
+    headers = {f for f in os.listdir(Bd.CSRC) if f.endswith((".h", ".cuh"))} | {"nvfp4ss.h"}
+    assert headers | set(cu) <= inputs
