@@ -34,8 +34,13 @@
  *   I0 = code of floor_E4M3(s_base); candidate c: t = fl(y*fl(1/v_c)),
  *   q = RNE_E2M1(t) saturating at 6; loss L_c = sum w (y - q v_c)^2;
  *   argmin over the window with exact ties going to the lowest code.
- *   A block with m == 0, or any block when S is not a positive finite float
- *   with finite 1/S, gets scale code 0 and nibbles carrying only the sign of x.
+ *   Zero rule: a block with m == 0, a block whose m (NaN counted) is NaN,
+ *   infinite or at least 2^48, and every block when S is not a positive finite
+ *   float with finite 1/S, gets scale code 0 and nibbles carrying only the sign
+ *   of y, for every method.  With S from nvfp4_global_scale a finite input gives
+ *   m <= 6*fp8_div, so only NaN/inf inputs (or a caller's S more than 2^36 below
+ *   amax/(6 D)) reach the 2^48 bound; below it every fp32 loss the kernels
+ *   accumulate stays finite for WMSE weights that are finite, >= 0 and <= 2^24.
  */
 #ifndef NVFP4SS_H
 #define NVFP4SS_H

@@ -27,6 +27,10 @@
  *                         t_i = fl32(y_i * r_c),  q_i = RNE_E2M1(t_i) (|t|>6 -> 6),
  *                         L_c = sum_i w_i (y_i - q_i*v_c)^2   in float64
  *   argmin over the window, exact ties -> lowest code.
+ *   Zero rule: a block with m == 0, a block holding a NaN, or whose m is
+ *   infinite or >= 2^48, and every block when S or fl32(1/S) is unusable, gets
+ *   scale code 0 and nibbles carrying only the sign of y (the paper defines no
+ *   output for these; the bound keeps fp32 losses finite on the GPU side).
  * The code decisions (q_i, I0, AbsMax rounding) are taken in float32, the
  * precision the GPU kernels decide in; losses are accumulated in float64.
  * Float ops here must not be contracted into FMAs: build with -ffp-contract=off.
@@ -211,18 +215,21 @@ int oracle_quantize(int method, const float* x, int64_t rows, int64_t cols, int 
         float y[64];
         uint8_t q[64], qbest[64];
         float m = 0.0f;
+        int has_nan = 0;
         for (int i = 0; i < block; i++) {
             y[i] = usable ? xb[i] * E : xb[i];
             float a = fabsf(y[i]);
-            if (a > m) m = a;
+            if (isnan(a)) has_nan = 1;
+            else if (a > m) m = a;
         }
         int chosen = 0;
         double Lbest = INFINITY, Lsecond = INFINITY;
         int clo = 0, chi = -1;
-        if (!usable || m == 0.0f) {
-            /* Zero block (or unusable S): scale 0, nibbles keep the sign of zero. */
+        for (int i = 0; i < block; i++) qbest[i] = signbit(y[i]) ? 8 : 0;
+        if (!usable || m == 0.0f || has_nan || !(m < 0x1p48f)) {
+            /* Zero rule (zero, non-finite or out-of-range block, or unusable S):
+             * scale 0, nibbles keep only the sign. */
             chosen = 0;
-            for (int i = 0; i < block; i++) qbest[i] = signbit(y[i]) ? 8 : 0;
             Lbest = 0.0;
             if (objective == ORACLE_WMSE) {
                 Lbest = 0.0;

@@ -16,14 +16,8 @@ __global__ void swizzle_pad_kernel(uint8_t* sf, int64_t rows, int64_t kb, int64_
 
 template <int DT, int METHOD, int OBJ, int BLOCK, int FIX>
 static cudaError_t launch_one(const QuantParams& p, int sms, cudaStream_t s) {
-    static int occ = 0;
-    if (!occ) {
-        int b = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, quantize_kernel<DT, METHOD, OBJ, BLOCK, FIX, 0>, 256,
-                                                          0) != cudaSuccess || b < 1)
-            b = 1;
-        occ = b;
-    }
+    static std::atomic<int> occ_cache[kOccDevices];
+    const int occ = occupancy_per_sm(occ_cache, quantize_kernel<DT, METHOD, OBJ, BLOCK, FIX, 0>, 256);
     const int64_t threads_needed = (p.nseg + 31) & ~(int64_t)31;
     int64_t grid = (threads_needed + 255) / 256;
     const int64_t cap = (int64_t)sms * occ;

@@ -8,14 +8,8 @@ namespace nvfp4 {
 
 template <int DT, int METHOD, int OBJ, int BLOCK, int FIX>
 static cudaError_t launch_dyn(const QuantParams& p_in, int sms, cudaStream_t s) {
-    static int occ = 0;
-    if (!occ) {
-        int b = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, quantize_kernel<DT, METHOD, OBJ, BLOCK, FIX, 1>, 256,
-                                                          0) != cudaSuccess || b < 1)
-            b = 1;
-        occ = b;
-    }
+    static std::atomic<int> occ_cache[kOccDevices];
+    const int occ = occupancy_per_sm(occ_cache, quantize_kernel<DT, METHOD, OBJ, BLOCK, FIX, 1>, 256);
     QuantParams p = p_in;
     int64_t grid = (p.nseg + 255) / 256;
     if (grid > (int64_t)sms * occ) grid = (int64_t)sms * occ;   // every CTA resident: the barrier can complete

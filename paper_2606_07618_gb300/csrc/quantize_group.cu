@@ -189,7 +189,7 @@ __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand*
             wkey = wp;
         }
     }
-    const bool zero = !usable || !(m > 0.0f);
+    const bool zero = zero_block(usable, m);
     float best = __int_as_float(0x7f800000);
     const int I0 = e4m3_floor_code(__fdiv_rn(m, 6.0f));
     const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
@@ -352,16 +352,8 @@ namespace {
 template <int DT, int OBJ, int DYN>
 cudaError_t launch_group(const GroupParams& p, int sms, cudaStream_t s) {
     constexpr int SW = kSweepThreads, threads = DYN ? kSweepThreads + 32 : kSweepThreads;
-    static std::atomic<int> occ{0};
-    if (!occ.load()) {
-        int b = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, quantize_group_kernel<DT, OBJ, DYN>, threads, 0) !=
-                cudaSuccess ||
-            b < 1)
-            b = 1;
-        occ.store(b);
-    }
-    const int64_t cap = (int64_t)sms * occ.load();
+    static std::atomic<int> occ_cache[kOccDevices];
+    const int64_t cap = (int64_t)sms * occupancy_per_sm(occ_cache, quantize_group_kernel<DT, OBJ, DYN>, threads);
     int64_t grid = (p.total_seg + SW - 1) / SW;
     if (grid > cap) {
         grid = cap;                                              // resident grid: every wait can complete

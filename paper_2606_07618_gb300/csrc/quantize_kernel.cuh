@@ -23,10 +23,30 @@
 // windows run a fixed, fully unrolled loop over [I0+lo, I0+hi] with no clamping
 // (those windows always contain a real code).  Custom windows clamp instead.
 #pragma once
+#include <atomic>
+
 #include "nvfp4_device.cuh"
 #include "nvfp4_kernels.h"
 
 namespace nvfp4 {
+
+// Resident CTAs per SM of `kernel` launched with `threads` threads on the
+// current device, looked up once per device; the per-device atomics make
+// first calls from several host threads safe.
+constexpr int kOccDevices = 64;
+template <typename K>
+inline int occupancy_per_sm(std::atomic<int> (&cache)[kOccDevices], K kernel, int threads) {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) dev = -1;
+    if (dev >= 0 && dev < kOccDevices) {
+        const int c = cache[dev].load(std::memory_order_relaxed);
+        if (c > 0) return c;
+    }
+    int b = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, kernel, threads, 0) != cudaSuccess || b < 1) b = 1;
+    if (dev >= 0 && dev < kOccDevices) cache[dev].store(b, std::memory_order_relaxed);
+    return b;
+}
 
 struct Cand {
     float r;        // fl(1/v_c)
@@ -70,10 +90,27 @@ __device__ __forceinline__ void load_raw(const void* x, int64_t g, Raw& r) {
     }
 }
 
+// NaN-propagating maxima: the block max is NaN if any element is NaN, so a
+// block holding a non-finite value is recognised from m alone (zero_block).
 __device__ __forceinline__ float max3f(float a, float b, float c) {
     float d;
-    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    asm("max.NaN.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
     return d;
+}
+__device__ __forceinline__ float max2f(float a, float b) {
+    float d;
+    asm("max.NaN.f32 %0, %1, %2;" : "=f"(d) : "f"(a), "f"(b));
+    return d;
+}
+
+// Blocks whose largest normalised magnitude m is NaN, infinite or >= 2^48
+// take the zero rule (scale code 0, nibbles carry only the signs), as do
+// all-zero blocks.  With S = amax/(6 D) every finite input gives m <= 6 D, so
+// only non-finite inputs or a caller-supplied S far below the tensor's own
+// reach it; below it every fp32 candidate loss stays finite for weights up to
+// 2^24 (16..64 terms of at most 2^24 * (2^48 + 2688)^2).
+__device__ __forceinline__ bool zero_block(bool usable, float m) {
+    return !usable || !(m > 0.0f && m < 281474976710656.0f);
 }
 
 // The segment's 16 inputs as 8 packed pairs y = fl(x*E) (one f32x2 multiply
@@ -103,7 +140,7 @@ __device__ __forceinline__ float raw_to_y(const Raw& r, u64 E2, u64 (&y2)[8]) {
         av[2 * j] = fabsf(a);
         av[2 * j + 1] = fabsf(b);
     }
-    // three-input max tree (NaNs are skipped, as by fmaxf)
+    // three-input max tree (a NaN element makes m NaN)
     const float p0 = max3f(av[0], av[1], av[2]), p1 = max3f(av[3], av[4], av[5]), p2 = max3f(av[6], av[7], av[8]);
     const float p3 = max3f(av[9], av[10], av[11]), p4 = max3f(av[12], av[13], av[14]);
     return max3f(max3f(p0, p1, p2), max3f(p3, p4, av[15]), 0.0f);
@@ -136,8 +173,8 @@ __device__ __forceinline__ float group_sum(float v) {
 }
 template <int SEGS>
 __device__ __forceinline__ float group_max(float v) {
-    if (SEGS >= 2) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 1));
-    if (SEGS >= 4) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 2));
+    if (SEGS >= 2) v = max2f(v, __shfl_xor_sync(0xffffffffu, v, 1));
+    if (SEGS >= 4) v = max2f(v, __shfl_xor_sync(0xffffffffu, v, 2));
     return v;
 }
 
@@ -362,7 +399,7 @@ __global__ void __launch_bounds__(256, quantize_min_blocks<METHOD, DT>()) quanti
             }
         }
 
-        const bool zero = !usable || !(m > 0.0f);
+        const bool zero = zero_block(usable, m);
         float best = __int_as_float(0x7f800000);
         int bestc = 0;
         if (METHOD == 0) {

@@ -79,6 +79,12 @@ def test_validation_without_gpu(L):
     assert L.nvfp4_global_scale(FAKE + 2, 0, 100, ctypes.c_float(256.0), FAKE + 4096, None, FAKE + 8192, 1 << 20,
                                 None) == 3
     assert L.nvfp4_global_scale(FAKE, 0, 100, ctypes.c_float(256.0), FAKE + 4096, None, FAKE + 8192, 16, None) == 1
+    # the allocation-free global scale refuses inputs past its static scratch
+    # (2^29 bf16 / 2^28 fp32 elements) on the host, before any CUDA call
+    for dt, n in ((0, (1 << 29) + 1), (1, (1 << 28) + 1)):
+        assert L.nvfp4_global_scale_noalloc(FAKE, dt, n, ctypes.c_float(256.0), FAKE + 4096, None, None) == 4
+    assert L.nvfp4_global_scale_noalloc(FAKE + 2, 0, 100, ctypes.c_float(256.0), FAKE + 4096, None, None) == 3
+    assert L.nvfp4_global_scale_noalloc(FAKE, 0, 100, ctypes.c_float(0.0), FAKE + 4096, None, None) == 1
     assert L.nvfp4_dequantize(FAKE, FAKE + 4096, 2, FAKE + 8192, 4, 64, 32, FAKE + 16384, 1, None) == 2
     assert L.nvfp4_dequantize(FAKE, FAKE + 4096, 3, FAKE + 8192, 4, 64, 16, FAKE + 16384, 1, None) == 1
     assert L.nvfp4_dequantize(FAKE, FAKE + 4096, 1, FAKE + 8192, 4, 64, 16, FAKE + 8, 1, None) == 3

@@ -34,6 +34,9 @@ MUTATIONS = [
      [F.test_e4m3_facts]),
     ("swizzle-transposed", "(r % 32) * 16 + ((r / 32) % 4) * 4", "(r % 32) * 4 + ((r / 32) % 4) * 16",
      [lambda o: SW.test_swizzle_layout_structure(o, 256, 8)]),
+    ("nan-block-swept", "if (isnan(a)) has_nan = 1;", "if (isnan(a)) has_nan = 0;",
+     [SW.test_nonfinite_and_out_of_range_blocks]),
+    ("no-2^48-bound", "!(m < 0x1p48f)", "!(m < INFINITY)", [SW.test_nonfinite_and_out_of_range_blocks]),
     ("opt-scale-wrong-midpoint", "{0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0}", "{0.25, 0.75, 1.25, 1.75, 2.5, 3.0, 5.0}",
      [SW.test_opt_scale_against_dense_scan]),
 ]

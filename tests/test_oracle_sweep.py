@@ -298,6 +298,53 @@ def test_zero_blocks_and_zero_tensor(oracle_mod):
     assert o["codes"][0, 1] == 0x80 and np.count_nonzero(o["codes"]) == 1
 
 
+def test_nonfinite_and_out_of_range_blocks(oracle_mod):
+    """Zero rule for non-finite and out-of-range blocks (a reading: the paper
+    defines no output for them).  Every other block must come out exactly as
+    in the clean tensor (blocks are independent given S, Sec. 4.2.1), and a
+    block just below the 2^48 bound is swept normally -- the exact-rational
+    brute force agrees with it."""
+    x = _mixed_inputs(4, 64, 71)[1].copy()
+    S, _ = oracle_mod.global_scale(x, 256.0)
+    Sf = np.float32(S)
+    E = np.float32(1) / Sf
+    xp = x.copy()
+    xp[0, 16 + 5] = np.nan
+    xp[1, 7] = np.inf
+    xp[2, 32 + 2] = -np.inf
+    xp[2, 32 + 3] = -0.0
+    big = np.float32(2.0 ** 48)
+    xp[3, 16 + 9] = np.float32(big / E)          # y = fl(x E) lands on or above 2^48
+    while np.float32(xp[3, 16 + 9] * E) < big:
+        xp[3, 16 + 9] = np.nextafter(xp[3, 16 + 9], np.float32(np.inf))
+    xp[3, 48 + 4] = np.float32(2.0 ** 47 / E)    # y around 2^47: swept normally
+    planted = {(0, 1), (1, 0), (2, 2), (3, 1)}
+    y_planted = (xp * E).astype(np.float32)
+    for method in (0, 1, 2):
+        for objective in (0, 1):
+            w = np.exp(np.random.default_rng(3).standard_normal(64)).astype(np.float32) if objective else None
+            ref = oracle_mod.quantize(method, x, 16, S, objective, w=w)
+            got = oracle_mod.quantize(method, xp, 16, S, objective, w=w)
+            for r in range(4):
+                for k in range(4):
+                    nib = [(got["codes"][r, 8 * k + j // 2] >> (4 * (j % 2))) & 0xF for j in range(16)]
+                    if (r, k) in planted:
+                        assert got["sf"][r, k] == 0, (method, objective, r, k)
+                        want = [8 if math.copysign(1.0, float(v)) < 0 else 0 for v in y_planted[r, 16 * k:16 * k + 16]]
+                        assert nib == want, (method, objective, r, k)
+                    elif (r, k) != (3, 3):
+                        assert got["sf"][r, k] == ref["sf"][r, k]
+                        assert np.array_equal(got["codes"][r, 8 * k:8 * k + 8], ref["codes"][r, 8 * k:8 * k + 8])
+            # the 2^47 block is an ordinary block: saturating scales, no zero rule
+            assert got["sf"][3, 3] >= 119
+            if method == 0:
+                wb = None if w is None else w[48:64]
+                bc, _, bq = _brute_block(xp[3, 48:64], S, wb, *oracle_mod.default_window(objective, 16))
+                assert got["sf"][3, 3] == bc
+                nib = [(got["codes"][3, 24 + j // 2] >> (4 * (j % 2))) & 0xF for j in range(16)]
+                assert nib == bq
+
+
 def test_global_scale_planted_max(oracle_mod):
     rng = np.random.default_rng(12)
     x = rng.uniform(-1, 1, 100003).astype(np.float32)
