@@ -37,6 +37,12 @@ MUTATIONS = [
     ("nan-block-swept", "if (isnan(a)) has_nan = 1;", "if (isnan(a)) has_nan = 0;",
      [SW.test_nonfinite_and_out_of_range_blocks]),
     ("no-2^48-bound", "!(m < 0x1p48f)", "!(m < INFINITY)", [SW.test_nonfinite_and_out_of_range_blocks]),
+    ("fp8-opt-floor-only", "if (Lc < Lf) { *code = ce;", "if (0) { *code = ce;",
+     [SW.test_fp8_quantised_optimum_picks_better_of_floor_and_ceil]),
+    ("fp8-opt-ceil-only", "if (Lc < Lf) { *code = ce;", "if (1) { *code = ce;",
+     [SW.test_fp8_quantised_optimum_picks_better_of_floor_and_ceil]),
+    ("fp8-opt-ties-to-ceil", "if (Lc < Lf) { *code = ce;", "if (Lc <= Lf) { *code = ce;",
+     [SW.test_fp8_quantised_optimum_picks_better_of_floor_and_ceil]),
     ("opt-scale-wrong-midpoint", "{0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0}", "{0.25, 0.75, 1.25, 1.75, 2.5, 3.0, 5.0}",
      [SW.test_opt_scale_against_dense_scan]),
 ]

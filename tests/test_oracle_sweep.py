@@ -244,6 +244,69 @@ def test_optimal_fp32_scale_lower_bounds_every_fp8_result(oracle_mod):
                         assert ss["best"][b] <= L8 * (1 + 1e-12)
 
 
+def _exact_loss_at(y, w, c):
+    """Exact-rational loss of scale code c on the float32 block y, with the
+    float32 rounding decisions of the contract (independent of the oracle)."""
+    v = bounds.E4M3[c][1]
+    r = np.float32(1) / np.float32(float(v))
+    L = Fraction(0)
+    for i, yi in enumerate(np.asarray(y, np.float32)):
+        t = np.float32(yi * r)
+        g, _ = _rne_mag(t)
+        wi = Fraction(float(w[i])) if w is not None else Fraction(1)
+        e = Fraction(float(yi)) - (g if t >= 0 else -g) * v
+        L += wi * e * e
+    return L
+
+
+def _floor_ceil_codes(s):
+    """floor_E4M3 / ceil_E4M3 of a positive real s as codes in 1..126, from the
+    exact value table (floor clamped up to code 1, ceil down to code 126)."""
+    sf = Fraction(s)
+    fl = max([c for c, v in bounds.E4M3 if c >= 1 and v <= sf], default=1)
+    ce = min([c for c, v in bounds.E4M3 if c >= 1 and v >= sf], default=126)
+    return fl, ce
+
+
+def test_fp8_quantised_optimum_picks_better_of_floor_and_ceil(oracle_mod):
+    """Appendix C's FP8-quantised optimum: of floor_E4M3(s*) and ceil_E4M3(s*)
+    the one with the lower loss, ties to the floor.  Checked against the exact
+    E4M3 table and exact-rational losses on sampled blocks of every
+    distribution, then on three constructed blocks where the ceiling is
+    strictly better, the floor is strictly better, and the two tie."""
+    rng = np.random.default_rng(12)
+    picked = {"floor": 0, "ceil": 0, "same": 0}
+    for x in _mixed_inputs(8, 128, 91):
+        S, _ = oracle_mod.global_scale(x, 256.0)
+        E = np.float32(1) / np.float32(S)
+        y = (x * E).astype(np.float32).reshape(-1, 16)
+        for b in rng.choice(y.shape[0], 12, replace=False):
+            for objective in (0, 1):
+                w = np.exp(rng.standard_normal(16)).astype(np.float32) if objective else None
+                s_opt, _ = oracle_mod.opt_scale(y[b], w)
+                code, L = oracle_mod.fp8_opt_code(y[b], w, s_opt)
+                fl, ce = _floor_ceil_codes(s_opt)
+                Lf, Lc = _exact_loss_at(y[b], w, fl), _exact_loss_at(y[b], w, ce)
+                want = ce if Lc < Lf else fl
+                picked["same" if fl == ce else ("ceil" if want == ce else "floor")] += 1
+                assert code == want, (b, objective, fl, ce, float(Lf), float(Lc))
+                assert abs(L - float(min(Lf, Lc))) <= 1e-12 * float(min(Lf, Lc)) + 1e-300
+    assert picked["floor"] > 0 and picked["ceil"] > 0
+    # constructed: s* = 1.05 lies between code 56 (1.0) and code 57 (1.125)
+    spike = np.zeros(16, np.float32)
+    spike[3] = 6.75                              # 6 * 1.125: exact at the ceiling, 0.75 off at the floor
+    assert oracle_mod.fp8_opt_code(spike, None, 1.05) == (57, 0.0)
+    spike[3] = 6.0                               # exact at the floor, 0.75 off at the ceiling
+    assert oracle_mod.fp8_opt_code(spike, None, 1.05) == (56, 0.0)
+    spike[3] = 1e-3                              # rounds to 0 under both: equal losses -> the floor
+    code, L = oracle_mod.fp8_opt_code(spike, None, 1.05)
+    assert code == 56 and L == float(np.float32(1e-3)) ** 2
+    # s* on a code, below the smallest code and above the largest
+    assert oracle_mod.fp8_opt_code(spike, None, 1.0)[0] == 56
+    assert oracle_mod.fp8_opt_code(spike, None, 2.0 ** -11)[0] == 1
+    assert oracle_mod.fp8_opt_code(spike, None, 500.0)[0] == 126
+
+
 # --------------------------------------------------------------------------- closed forms
 def test_single_spike_block(oracle_mod):
     for code, sign in ((58, 1.0), (58, -1.0), (40, 1.0), (90, -1.0)):
