@@ -212,12 +212,14 @@ size_t scalesweep_quantize_group_workspace(void);
 /*
  * ScaleSweep quantisation of `count` tensors (1..NVFP4_GROUP_MAX, e.g. all
  * linear weights of one transformer layer) in one launch: for every tensor the
- * result of scalesweep_quantize with block 16 and the default window ([-3, 7]
- * MSE, [-8, 7] WMSE, Sec. 4.2.2), bit for bit.  The segments of all tensors are
- * walked by one grid, so the call has a single launch tail instead of one per
- * tensor.
+ * result of scalesweep_quantize with the same block and the default window
+ * ([-3, 7] MSE with block 16, [-8, 7] otherwise, Sec. 4.2.2), bit for bit.  The
+ * segments of all tensors are walked by one grid, so the call has a single
+ * launch tail instead of one per tensor.
  *   tensors     host array of `count` descriptors, read during the call only.
  *   dt, obj     input type and objective, shared by all tensors.
+ *   block       16, 32 or 64, shared by all tensors (every cols % block == 0);
+ *               sf_swizzled only with block 16.
  *   fp8_div     0: static global scales, S[i] is read for tensor i.
  *               > 0: per-call (dynamic) global scales, S[i] = fl32(amax_i /
  *               fl32(6*fp8_div)) over tensor i (Sec. 4.2.1) is computed in the
@@ -234,9 +236,21 @@ size_t scalesweep_quantize_group_workspace(void);
  * Outputs must not overlap any input, S, status_dev, the workspace or each
  * other.  Concurrent calls must use distinct workspaces.
  */
-nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt,
+nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt, int block,
                                        nvfp4_objective obj, float fp8_div, float* S, int* status_dev,
                                        void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * AbsMax quantisation (Sec. 3.2, as absmax_quantize) of `count` tensors in one
+ * launch, with static or in-launch global scales exactly as
+ * scalesweep_quantize_group (same descriptors, arguments, workspace and
+ * status word; the descriptors' w and w_row_stride are not read).  The
+ * baseline the grouped sweep's overhead is measured against, launch shape for
+ * launch shape.
+ */
+nvfp4_status absmax_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt, int block,
+                                   float fp8_div, float* S, int* status_dev, void* workspace, size_t ws_bytes,
+                                   void* stream);
 
 /*
  * Self-test of the bounded device waits (failure detection; the paper has no

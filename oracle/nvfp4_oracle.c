@@ -380,6 +380,9 @@ int oracle_dequantize(const uint8_t* codes, const uint8_t* sf, int layout, float
 {
     if (block <= 0 || cols % block != 0 || cols % 2 != 0) return -1;
     int64_t kb = cols / block;
+#ifdef _OPENMP
+#pragma omp parallel for schedule(static)
+#endif
     for (int64_t r = 0; r < rows; r++) {
         for (int64_t j = 0; j < cols; j++) {
             int64_t k = j / block;

@@ -69,7 +69,8 @@ def lib() -> ctypes.CDLL:
         L.scalesweep_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, i, p, i64, i, i, p, p, p, sz, p, p, p, p, p]
         L.absmax_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, p, p, p, sz, p, p, p, p, p]
         L.scalesweep_quantize_group_workspace.argtypes, L.scalesweep_quantize_group_workspace.restype = [], sz
-        L.scalesweep_quantize_group.argtypes = [ctypes.POINTER(GroupTensor), i, i, i, f, p, p, p, sz, p]
+        L.scalesweep_quantize_group.argtypes = [ctypes.POINTER(GroupTensor), i, i, i, i, f, p, p, p, sz, p]
+        L.absmax_quantize_group.argtypes = [ctypes.POINTER(GroupTensor), i, i, i, f, p, p, p, sz, p]
         L.nvfp4_selftest_wait_timeout.argtypes = [i, p, i64, i64, p, p, p, sz, p, p, p]
         L.nvfp4_optimal_scale.argtypes = [p, i, i64, i64, i, p, i, p, i64, p, p, p, p, p]
         L.nvfp4_ldlq_prepare_workspace.argtypes, L.nvfp4_ldlq_prepare_workspace.restype = [i64], sz
@@ -79,7 +80,7 @@ def lib() -> ctypes.CDLL:
         for fn in ("nvfp4_global_scale", "nvfp4_global_scale_noalloc", "scalesweep_quantize", "absmax_quantize",
                    "four_over_six_quantize", "nvfp4_dequantize", "scalesweep_quantize_dynamic",
                    "absmax_quantize_dynamic", "nvfp4_optimal_scale", "nvfp4_ldlq_prepare", "ldlq_quantize",
-                   "scalesweep_quantize_group", "nvfp4_selftest_wait_timeout"):
+                   "scalesweep_quantize_group", "absmax_quantize_group", "nvfp4_selftest_wait_timeout"):
             getattr(L, fn).restype = i
         _lib = L
     return _lib
@@ -207,13 +208,23 @@ def group_descriptors(xs, ws, w_row_strides, codes, sf_linear, sf_swizzled):
 
 
 def scalesweep_quantize_group(desc, dtype: int, objective: int, fp8_div: float, S, status=None, workspace=None,
-                              stream=None):
+                              stream=None, block: int = 16):
     """desc: the array from group_descriptors.  fp8_div 0 reads S[i]; > 0
     computes and writes S[i] in the launch."""
     ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
-    rc = lib().scalesweep_quantize_group(desc, len(desc), int(dtype), int(objective), float(fp8_div), _ptr(S),
-                                         _ptr(status), _ptr(workspace), ws_bytes, _stream(stream))
+    rc = lib().scalesweep_quantize_group(desc, len(desc), int(dtype), int(block), int(objective), float(fp8_div),
+                                         _ptr(S), _ptr(status), _ptr(workspace), ws_bytes, _stream(stream))
     _check("scalesweep_quantize_group", rc)
+
+
+def absmax_quantize_group(desc, dtype: int, fp8_div: float, S, status=None, workspace=None, stream=None,
+                          block: int = 16):
+    """AbsMax over the tensors of desc in one launch (static or in-launch scales,
+    as scalesweep_quantize_group)."""
+    ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    rc = lib().absmax_quantize_group(desc, len(desc), int(dtype), int(block), float(fp8_div), _ptr(S),
+                                     _ptr(status), _ptr(workspace), ws_bytes, _stream(stream))
+    _check("absmax_quantize_group", rc)
 
 
 def nvfp4_selftest_wait_timeout(which: int, x, S, status, workspace, codes, sf_linear, stream=None):

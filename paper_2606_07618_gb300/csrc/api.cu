@@ -278,12 +278,15 @@ static_assert(kGroupMax == NVFP4_GROUP_MAX, "group descriptor count");
 size_t scalesweep_quantize_group_workspace(void) { return kGroupWorkspace; }
 
 namespace {
-nvfp4_status group_common(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt, nvfp4_objective obj,
-                          float fp8_div, float* S, int* status_dev, void* workspace, size_t ws_bytes, void* stream,
-                          unsigned wait_extra) {
+// method 0 ScaleSweep (objective obj), 1 AbsMax (obj ignored: MSE, no weights read).
+nvfp4_status group_common(int method, const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt, int block,
+                          nvfp4_objective obj, float fp8_div, float* S, int* status_dev, void* workspace,
+                          size_t ws_bytes, void* stream, unsigned wait_extra) {
     if (dt != NVFP4_IN_BF16 && dt != NVFP4_IN_F32) return NVFP4_ERR_INVALID_ARG;
+    if (method == 1) obj = NVFP4_OBJ_MSE;
     if (obj != NVFP4_OBJ_MSE && obj != NVFP4_OBJ_WMSE) return NVFP4_ERR_INVALID_ARG;
     if (!tensors || count < 1 || count > NVFP4_GROUP_MAX || !S) return NVFP4_ERR_INVALID_ARG;
+    if (block != 16 && block != 32 && block != 64) return NVFP4_ERR_UNSUPPORTED;
     const bool dyn = fp8_div != 0.0f;
     if (dyn && (!(fp8_div > 0.0f) || fp8_div > 1e30f)) return NVFP4_ERR_INVALID_ARG;
     if (dyn && (!workspace || ws_bytes < kGroupWorkspace)) return NVFP4_ERR_INVALID_ARG;
@@ -308,8 +311,9 @@ nvfp4_status group_common(const nvfp4_group_tensor* tensors, int count, nvfp4_dt
     Shape sh[NVFP4_GROUP_MAX];
     for (int i = 0; i < count; i++) {
         const nvfp4_group_tensor& t = tensors[i];
-        nvfp4_status st = check_shape(t.rows, t.cols, 16, &sh[i]);
+        nvfp4_status st = check_shape(t.rows, t.cols, block, &sh[i]);
         if (st != NVFP4_OK) return st;
+        if (t.sf_swizzled && block != 16) return NVFP4_ERR_UNSUPPORTED;
         if (sh[i].n == 0) continue;
         if (!t.x || !t.codes || (!t.sf_linear && !t.sf_swizzled)) return NVFP4_ERR_INVALID_ARG;
         if (!aligned(t.x, 16) || !aligned(t.codes, 8)) return NVFP4_ERR_ALIGNMENT;
@@ -392,16 +396,24 @@ nvfp4_status group_common(const nvfp4_group_tensor* tensors, int count, nvfp4_dt
     p.amax_bits = dyn ? static_cast<unsigned*>(workspace) : nullptr;
     p.arrived = dyn ? static_cast<unsigned*>(workspace) + kGroupMax : nullptr;
     p.wait_extra = wait_extra;
-    const cudaError_t e = launch_quantize_group(p, rows, dt == NVFP4_IN_BF16 ? 0 : 1, obj == NVFP4_OBJ_WMSE ? 1 : 0,
-                                                sms, static_cast<cudaStream_t>(stream));
+    const cudaError_t e = launch_quantize_group(p, rows, dt == NVFP4_IN_BF16 ? 0 : 1, method,
+                                                obj == NVFP4_OBJ_WMSE ? 1 : 0, block, sms,
+                                                static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
 }
 }  // namespace
 
-nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt,
+nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt, int block,
                                        nvfp4_objective obj, float fp8_div, float* S, int* status_dev,
                                        void* workspace, size_t ws_bytes, void* stream) {
-    return group_common(tensors, count, dt, obj, fp8_div, S, status_dev, workspace, ws_bytes, stream, 0);
+    return group_common(0, tensors, count, dt, block, obj, fp8_div, S, status_dev, workspace, ws_bytes, stream, 0);
+}
+
+nvfp4_status absmax_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt, int block,
+                                   float fp8_div, float* S, int* status_dev, void* workspace, size_t ws_bytes,
+                                   void* stream) {
+    return group_common(1, tensors, count, dt, block, NVFP4_OBJ_MSE, fp8_div, S, status_dev, workspace, ws_bytes,
+                        stream, 0);
 }
 
 nvfp4_status nvfp4_selftest_wait_timeout(int which, const void* x, int64_t rows, int64_t cols, float* S,
@@ -415,7 +427,8 @@ nvfp4_status nvfp4_selftest_wait_timeout(int which, const void* x, int64_t rows,
                                &d);
     }
     const nvfp4_group_tensor t{x, rows, cols, nullptr, 0, codes, sf_linear, nullptr};
-    return group_common(&t, 1, NVFP4_IN_BF16, NVFP4_OBJ_MSE, 256.0f, S, status_dev, workspace, ws_bytes, stream, 1);
+    return group_common(0, &t, 1, NVFP4_IN_BF16, 16, NVFP4_OBJ_MSE, 256.0f, S, status_dev, workspace, ws_bytes,
+                        stream, 1);
 }
 
 nvfp4_status absmax_quantize_dynamic(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,

@@ -48,10 +48,11 @@ constexpr size_t kGroupWorkspace = 256;   // amax_bits + arrived for kGroupMax t
 // straddles two tensors.
 constexpr int kGroupCtaSegments = 256;
 
-// dtype 0 bf16 / 1 f32; obj 0 MSE / 1 WMSE.  Zeroes the workspace counters
-// (dyn), launches the grouped kernel (cooperative when dyn) and the swizzle pad
+// dtype 0 bf16 / 1 f32; method 0 ScaleSweep / 1 AbsMax; obj 0 MSE / 1 WMSE
+// (ScaleSweep only); block 16/32/64.  Zeroes the workspace counters (dyn),
+// launches the grouped kernel (cooperative when dyn) and the swizzle pad
 // kernels for shapes that need them.
-cudaError_t launch_quantize_group(const GroupParams& p, const int64_t* rows, int dtype, int obj, int sms,
-                                  cudaStream_t s);
+cudaError_t launch_quantize_group(const GroupParams& p, const int64_t* rows, int dtype, int method, int obj,
+                                  int block, int sms, cudaStream_t s);
 
 }  // namespace nvfp4

@@ -1,6 +1,7 @@
-// Grouped ScaleSweep (Sec. 4.2.2, default windows, block 16) over a list of
-// tensors in one launch, with each tensor's global scale (Sec. 4.2.1,
-// S = fl(amax / fl(6 D))) optionally reduced inside the same launch.
+// Grouped ScaleSweep (Sec. 4.2.2, default windows) or AbsMax (Sec. 3.2) over a
+// list of tensors in one launch, blocks of 16, 32 or 64 elements, with each
+// tensor's global scale (Sec. 4.2.1, S = fl(amax / fl(6 D))) optionally
+// reduced inside the same launch.
 //
 // Why: a transformer layer has tensors of very different sizes (k/v are 1/14
 // of gate/up/down in Llama-3-8B).  One launch per tensor pays a ramp-down tail
@@ -14,9 +15,10 @@
 // iteration; every tensor's segment range is padded to a multiple of 256, so
 // the tensor index t is CTA-uniform and the descriptor fields are read as
 // uniform kernel-parameter operands.  The per-segment sweep is the one of
-// quantize_kernel (FIX = 1, block 16): y = fl(x E), I0 from fl(m/6), the 11
-// (MSE) or 16 (WMSE) candidates of the poison-padded table, lowest-code
-// argmin, nibbles and both scale layouts.
+// quantize_kernel (FIX = 1): y = fl(x E), I0 from fl(m/6), the 11 (MSE, block
+// 16) or 16 candidates of the poison-padded table, lowest-code argmin, nibbles
+// and both scale layouts; blocks of 32/64 are 2/4 lanes combined by
+// xor-shuffles (a CTA's 256 segments always hold whole blocks).
 //
 // Reduction warp (a ninth warp per CTA, dynamic scales only).  The reduction
 // warps of the grid split every tensor's 16-byte input vectors round-robin
@@ -150,14 +152,19 @@ __device__ __forceinline__ void reduce_warp(const GroupParams& p, int lane) {
     }
 }
 
-// WMSE weights of the lane's segment are kept in w2 across iterations and
-// reloaded only when they come from another address (wkey): with a CTA stride
-// that is a multiple of the tensor's scale columns a lane keeps its column
-// block, so per-channel weights are loaded once per tensor.
-template <int DT, int OBJ>
+// One 16-element segment of the grid-stride loop: ScaleSweep (METHOD 0,
+// default window) or AbsMax (METHOD 1) for a block of BLOCK elements, which is
+// 1, 2 or 4 consecutive lanes (their maxima and losses combined by
+// xor-shuffles, as in quantize_kernel).  WMSE weights of the lane's segment
+// are kept in w2 across iterations and reloaded only when they come from
+// another address (wkey): with a CTA stride that is a multiple of the
+// tensor's segments per row a lane keeps its columns, so per-channel weights
+// are loaded once per tensor.
+template <int DT, int METHOD, int OBJ, int BLOCK>
 __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand* tab, const Raw& cur, int64_t g,
                                                bool valid, u64 E2, bool usable, u64 (&w2)[8], const float*& wkey) {
-    constexpr int FIX_LO = OBJ == 0 ? -3 : -8;
+    constexpr int SEGS = BLOCK / 16;
+    constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
     constexpr int FIX_K = 7 - FIX_LO + 1;
     u64 y2[8];
     float m = 0.0f;
@@ -167,18 +174,23 @@ __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand*
 #pragma unroll
         for (int j = 0; j < 8; j++) y2[j] = 0ull;
     }
-    if (OBJ == 1) {
-        int64_t row, kbi;
+    m = group_max<SEGS>(m);
+    const int64_t blk = g / SEGS;                           // scale-block index (g >= 0: a shift)
+    auto row_col = [&](int64_t& row, int64_t& kbi) {
         if (d.narrow) {
-            const uint32_t b32 = (uint32_t)g;
+            const uint32_t b32 = (uint32_t)blk;
             const uint32_t r32 = fast_div(b32, d.kb_div);
             row = r32;
             kbi = b32 - r32 * (uint32_t)d.kb;
         } else {
-            row = g / d.kb;
-            kbi = g - row * d.kb;
+            row = blk / d.kb;
+            kbi = blk - row * d.kb;
         }
-        const float* wp = d.w + row * d.w_row_stride + kbi * 16;
+    };
+    if (METHOD == 0 && OBJ == 1) {
+        int64_t row, kbi;
+        row_col(row, kbi);
+        const float* wp = d.w + row * d.w_row_stride + kbi * BLOCK + (g % SEGS) * 16;
         if (valid && wp != wkey) {
 #pragma unroll
             for (int j = 0; j < 4; j++) {
@@ -190,20 +202,25 @@ __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand*
         }
     }
     const bool zero = zero_block(usable, m);
-    float best = __int_as_float(0x7f800000);
-    const int I0 = e4m3_floor_code(__fdiv_rn(m, 6.0f));
-    const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
-    int bk = 0;
+    int bestc;
+    if (METHOD == 0) {
+        float best = __int_as_float(0x7f800000);
+        const int I0 = e4m3_floor_code(__fdiv_rn(m, 6.0f));
+        const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
+        int bk = 0;
 #pragma unroll
-    for (int k = 0; k < FIX_K; k++) {
-        const Cand cd = tb[k];
-        const float L = seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv);
-        if (L < best) {
-            best = L;
-            bk = k;
+        for (int k = 0; k < FIX_K; k++) {
+            const Cand cd = tb[k];
+            const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));
+            if (L < best) {
+                best = L;
+                bk = k;
+            }
         }
+        bestc = I0 + FIX_LO + bk;
+    } else {
+        bestc = max((int)e4m3_rn_code(__fdiv_rn(m, 6.0f)), 1);
     }
-    int bestc = I0 + FIX_LO + bk;
     uint32_t packed[2];
     if (zero) {
 #pragma unroll
@@ -235,19 +252,13 @@ __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand*
     }
     if (valid) {
         *reinterpret_cast<uint2*>(d.codes + g * 8) = make_uint2(packed[0], packed[1]);
-        if (d.sf_linear) d.sf_linear[g] = (uint8_t)bestc;
-        if (d.sf_swizzled) {
-            int64_t row, kbi;                                   // recomputed here: not live across the sweep
-            if (d.narrow) {
-                const uint32_t b32 = (uint32_t)g;
-                const uint32_t r32 = fast_div(b32, d.kb_div);
-                row = r32;
-                kbi = b32 - r32 * (uint32_t)d.kb;
-            } else {
-                row = g / d.kb;
-                kbi = g - row * d.kb;
+        if ((g % SEGS) == 0) {
+            if (d.sf_linear) d.sf_linear[blk] = (uint8_t)bestc;
+            if (BLOCK == 16 && d.sf_swizzled) {
+                int64_t row, kbi;                               // recomputed here: not live across the sweep
+                row_col(row, kbi);
+                d.sf_swizzled[swizzle_offset(row, kbi, d.kpad4)] = (uint8_t)bestc;
             }
-            d.sf_swizzled[swizzle_offset(row, kbi, d.kpad4)] = (uint8_t)bestc;
         }
     }
 }
@@ -265,7 +276,7 @@ __device__ __forceinline__ int tensor_at(const GroupParams& p, int t, int64_t se
 // scales reduced in the launch by a ninth warp per CTA.  (Nine warps cap the
 // registers at 96 per thread -- two CTAs put five warps on two schedulers --
 // which measured faster than seven sweep warps plus one reduction warp.)
-template <int DT, int OBJ, int DYN>
+template <int DT, int METHOD, int OBJ, int BLOCK, int DYN>
 __global__ void __launch_bounds__(DYN ? kSweepThreads + 32 : kSweepThreads, NVFP4_GROUP_MINB)
     quantize_group_kernel(const __grid_constant__ GroupParams p) {
     constexpr int SW = kSweepThreads;
@@ -338,7 +349,7 @@ __global__ void __launch_bounds__(DYN ? kSweepThreads + 32 : kSweepThreads, NVFP
                 const int64_t gn = nb + tid - p.t[tn].seg_begin;
                 if (gn < p.t[tn].nseg) load_raw<DT>(p.t[tn].x, gn, nxt);
             }
-            sweep_segments<DT, OBJ>(d, tab, cur, g, valid, E2, usable, w2, wkey);
+            sweep_segments<DT, METHOD, OBJ, BLOCK>(d, tab, cur, g, valid, E2, usable, w2, wkey);
             cur = nxt;
         }
         t = tensor_at(p, t, cbase);
@@ -349,21 +360,24 @@ __global__ void __launch_bounds__(DYN ? kSweepThreads + 32 : kSweepThreads, NVFP
 
 namespace {
 
-template <int DT, int OBJ, int DYN>
+template <int DT, int METHOD, int OBJ, int BLOCK, int DYN>
 cudaError_t launch_group(const GroupParams& p, int sms, cudaStream_t s) {
     constexpr int SW = kSweepThreads, threads = DYN ? kSweepThreads + 32 : kSweepThreads;
+    constexpr int SEGS = BLOCK / 16;
     static std::atomic<int> occ_cache[kOccDevices];
-    const int64_t cap = (int64_t)sms * occupancy_per_sm(occ_cache, quantize_group_kernel<DT, OBJ, DYN>, threads);
+    const int64_t cap = (int64_t)sms *
+                        occupancy_per_sm(occ_cache, quantize_group_kernel<DT, METHOD, OBJ, BLOCK, DYN>, threads);
     int64_t grid = (p.total_seg + SW - 1) / SW;
     if (grid > cap) {
         grid = cap;                                              // resident grid: every wait can complete
-        if (OBJ == 1) {
+        if (METHOD == 0 && OBJ == 1) {
             // Up to 1/32 fewer CTAs if that makes the CTA stride a multiple of
-            // more tensors' scale-column counts (lanes then keep their weights).
+            // more tensors' segments per row (lanes then keep their weights).
             auto covered = [&](int64_t g) {
                 int64_t c = 0;
                 for (int i = 0; i < p.count; i++)
-                    if (p.t[i].w_row_stride == 0 && p.t[i].kb > 0 && (g * SW) % p.t[i].kb == 0) c += p.t[i].nseg;
+                    if (p.t[i].w_row_stride == 0 && p.t[i].kb > 0 && (g * SW) % (p.t[i].kb * SEGS) == 0)
+                        c += p.t[i].nseg;
                 return c;
             };
             int64_t best = grid, best_c = covered(grid);
@@ -382,26 +396,40 @@ cudaError_t launch_group(const GroupParams& p, int sms, cudaStream_t s) {
         cudaError_t e = cudaMemsetAsync(p.amax_bits, 0, kGroupWorkspace, s);
         if (e != cudaSuccess) return e;
         void* args[] = {(void*)&p};
-        return cudaLaunchCooperativeKernel((const void*)quantize_group_kernel<DT, OBJ, 1>, dim3((unsigned)grid),
-                                           dim3(threads), args, 0, s);
+        return cudaLaunchCooperativeKernel((const void*)quantize_group_kernel<DT, METHOD, OBJ, BLOCK, 1>,
+                                           dim3((unsigned)grid), dim3(threads), args, 0, s);
     }
-    quantize_group_kernel<DT, OBJ, 0><<<(unsigned)grid, threads, 0, s>>>(p);
+    quantize_group_kernel<DT, METHOD, OBJ, BLOCK, 0><<<(unsigned)grid, threads, 0, s>>>(p);
     return cudaGetLastError();
+}
+
+template <int DT, int METHOD, int OBJ, int BLOCK>
+cudaError_t launch_dyn_or_static(const GroupParams& p, int sms, cudaStream_t s) {
+    return p.dyn ? launch_group<DT, METHOD, OBJ, BLOCK, 1>(p, sms, s) : launch_group<DT, METHOD, OBJ, BLOCK, 0>(p, sms, s);
+}
+
+template <int DT, int METHOD, int OBJ>
+cudaError_t launch_block(const GroupParams& p, int block, int sms, cudaStream_t s) {
+    switch (block) {
+        case 16: return launch_dyn_or_static<DT, METHOD, OBJ, 16>(p, sms, s);
+        case 32: return launch_dyn_or_static<DT, METHOD, OBJ, 32>(p, sms, s);
+        default: return launch_dyn_or_static<DT, METHOD, OBJ, 64>(p, sms, s);
+    }
+}
+
+template <int DT>
+cudaError_t launch_method(const GroupParams& p, int method, int obj, int block, int sms, cudaStream_t s) {
+    if (method == 1) return launch_block<DT, 1, 0>(p, block, sms, s);
+    return obj == 1 ? launch_block<DT, 0, 1>(p, block, sms, s) : launch_block<DT, 0, 0>(p, block, sms, s);
 }
 
 }  // namespace
 
-cudaError_t launch_quantize_group(const GroupParams& p, const int64_t* rows, int dtype, int obj, int sms,
-                                  cudaStream_t s) {
+cudaError_t launch_quantize_group(const GroupParams& p, const int64_t* rows, int dtype, int method, int obj,
+                                  int block, int sms, cudaStream_t s) {
     cudaError_t e = cudaSuccess;
     if (p.total_seg > 0 || p.dyn) {
-        if (p.dyn) {
-            if (dtype == 0) e = obj == 1 ? launch_group<0, 1, 1>(p, sms, s) : launch_group<0, 0, 1>(p, sms, s);
-            else e = obj == 1 ? launch_group<1, 1, 1>(p, sms, s) : launch_group<1, 0, 1>(p, sms, s);
-        } else {
-            if (dtype == 0) e = obj == 1 ? launch_group<0, 1, 0>(p, sms, s) : launch_group<0, 0, 0>(p, sms, s);
-            else e = obj == 1 ? launch_group<1, 1, 0>(p, sms, s) : launch_group<1, 0, 0>(p, sms, s);
-        }
+        e = dtype == 0 ? launch_method<0>(p, method, obj, block, sms, s) : launch_method<1>(p, method, obj, block, sms, s);
         if (e != cudaSuccess) return e;
     }
     for (int i = 0; i < p.count; i++) {

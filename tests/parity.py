@@ -35,19 +35,35 @@ def compare_quantize(x, S, block, objective, w, w_row_stride, gpu, ref, method=0
     diff = np.nonzero(g_sf != r_sf)[0]
     stats = {"blocks": r_sf.size, "near_tie_accepted": int(diff.size)}
     wn = None if w is None else to_np(w)
+    Lg = None
     if diff.size:
         best, second = ref["best"][diff], ref["second"][diff]
         gap_ok = (second - best) <= REL * np.abs(best)
         bad = diff[~gap_ok]
         assert bad.size == 0, (f"{bad.size} blocks differ beyond near-ties, e.g. block {bad[0]}: gpu {g_sf[bad[0]]} "
                                f"oracle {r_sf[bad[0]]} best {ref['best'][bad[0]]!r} second {ref['second'][bad[0]]!r}")
-        Lg, cg = oracle.block_losses_at(xs, block, S, g_sf, objective, w=wn, w_row_stride=w_row_stride,
-                                        want_codes=True)
+        # score the GPU's picks with the oracle, on the rows that hold them only
+        rows, cols = xs.shape
+        kb = cols // block
+        rsel = np.unique(diff // kb)
+        pos = np.searchsorted(rsel, diff // kb) * kb + diff % kb
+        if wn is None or w_row_stride == 0:
+            wsub = wn
+        else:                                           # per-element weights: the selected rows' strides
+            wf = wn.reshape(-1)
+            wsub = np.zeros((rsel.size, w_row_stride), np.float32)
+            for i, r in enumerate(rsel):
+                seg = wf[r * w_row_stride:(r + 1) * w_row_stride]
+                wsub[i, :seg.size] = seg
+        Ls, cs = oracle.block_losses_at(xs[rsel], block, S, g_sf.reshape(rows, kb)[rsel], objective, w=wsub,
+                                        w_row_stride=w_row_stride, want_codes=True)
+        Lg = np.full(r_sf.size, np.nan)
+        Lg[diff] = Ls[pos]
         assert np.all(Lg[diff] <= best * (1 + REL)), "GPU near-tie pick is not within 1e-6 of the best"
         # nibbles of differing blocks must match the oracle's nibbles for the GPU's scale
         cpb = block // 2
         gc = g_codes.reshape(-1, cpb)
-        assert np.array_equal(gc[diff], cg.reshape(-1, cpb)[diff])
+        assert np.array_equal(gc[diff], cs.reshape(-1, cpb)[pos])
         same = np.ones(r_sf.size, bool)
         same[diff] = False
         assert np.array_equal(gc[same], ref["codes"].reshape(-1, cpb)[same])

@@ -31,7 +31,7 @@ def test_header_declares_the_api():
         "nvfp4_dynamic_workspace", "scalesweep_quantize_dynamic", "absmax_quantize_dynamic",
         "nvfp4_optimal_scale", "nvfp4_ldlq_prepare_workspace", "nvfp4_ldlq_prepare", "nvfp4_ldlq_workspace",
         "ldlq_quantize", "scalesweep_quantize_group_workspace", "scalesweep_quantize_group",
-        "nvfp4_selftest_wait_timeout"])
+        "absmax_quantize_group", "nvfp4_selftest_wait_timeout"])
 
 
 def test_library_exports_every_declared_symbol(L):
@@ -123,7 +123,7 @@ def test_ldlq_validation_without_gpu(L):
 
 
 def test_group_validation_without_gpu(L):
-    """Argument checks of scalesweep_quantize_group that return before any CUDA
+    """Argument checks of scalesweep_quantize_group / absmax_quantize_group that return before any CUDA
     call (the overlap checks, which need device pointers to pass, are
     exercised with real buffers in the GPU tests)."""
     from paper_2606_07618_gb300 import binding as B
@@ -142,8 +142,10 @@ def test_group_validation_without_gpu(L):
         return arr
 
     S, st, ws = FAKE + 0x3000000, FAKE + 0x3000100, FAKE + 0x3001000
-    g = lambda d, n=2, dt=0, obj=0, div=256.0, S=S, ws=ws, wsb=256: \
-        L.scalesweep_quantize_group(d, n, dt, obj, f(div), S, st, ws, wsb, None)
+    g = lambda d, n=2, dt=0, obj=0, div=256.0, S=S, ws=ws, wsb=256, block=16: \
+        L.scalesweep_quantize_group(d, n, dt, block, obj, f(div), S, st, ws, wsb, None)
+    a = lambda d, n=2, dt=0, div=256.0, S=S, ws=ws, wsb=256, block=16: \
+        L.absmax_quantize_group(d, n, dt, block, f(div), S, st, ws, wsb, None)
     assert L.scalesweep_quantize_group_workspace() >= 128
     assert g(desc(), n=0) == 1                        # empty group
     assert g(desc(), n=17) == 1                       # more than NVFP4_GROUP_MAX
@@ -163,6 +165,14 @@ def test_group_validation_without_gpu(L):
     assert g(desc(every={"w": FAKE + 0x4000004}), obj=1) == 3
     assert g(desc(every={"w": FAKE + 0x4000000, "w_row_stride": 8}), obj=1) == 1
     assert g(desc({"rows": 2 ** 40, "cols": 2 ** 40})) == 4
+    assert g(desc(), block=8) == 2                    # block not in {16, 32, 64}
+    assert g(desc({"cols": 48}), block=32) == 1       # cols % block
+    assert g(desc({"sf_swizzled": FAKE + 0x5000000}), block=32) == 2   # swizzled scales need block 16
+    assert a(desc(), n=0) == 1
+    assert a(desc(), block=128) == 2
+    assert a(desc(), ws=None) == 1
+    assert a(desc({"x": FAKE + 2})) == 3
+    assert a(desc({"sf_swizzled": FAKE + 0x5000000}), block=64) == 2
     st_test = lambda which=0, status=st, rows=4: L.nvfp4_selftest_wait_timeout(
         which, FAKE, rows, 64, S, status, ws, 1 << 12, FAKE + 0x1000000, FAKE + 0x2000000, None)
     assert st_test(which=2) == 1

@@ -1,23 +1,35 @@
-"""Full-size parity on every synthetic workload, in the launch configuration
-bench.py times (whole tensors, default windows, both scale layouts).
+"""Full-size parity on every synthetic workload, every block, in the launch
+configuration bench.py times (paper_2606_07618_gb300.step: one grouped launch
+with in-launch global scales, or the fused dynamic launch for the activation).
 
-The GPU quantises each whole tensor; the oracle recomputes a sample of rows
-(first, last and evenly spread ones) with the same S; every other block is
-checked through properties that hold at any size (scale codes in the window
-range, swizzled = permuted linear, dequantised values bounded by the block's
-own scale).  The global scale is compared bit-exactly on the whole tensor.
+For every tensor of every workload -- the 2048x2048 weight, the Llama-3-8B
+layer, the 8192x4096 activation, K/V/Q, and both Qwen2.5-72B-shaped matrices
+at blocks 16/32/64 with MSE and WMSE:
+
+  * S equals the oracle's bit for bit;
+  * every block's scale and nibbles equal the oracle's, except on the
+    oracle's near-ties (best and second-best within 1e-6 relative), where the
+    GPU's pick must score within 1e-6 of the best and carry the oracle's
+    nibbles for that scale (tests/parity.py);
+  * the dequantised tensor equals the oracle's dequantisation of the same
+    codes bit for bit (swizzled scales for block 16, linear otherwise);
+  * the tensor's summed loss, measured on the GPU from its own output in the
+    x domain, agrees with the oracle's summed block optimum times S^2 to 1e-5.
+
+The per-workload counts (blocks checked, near-ties accepted) are printed.
 """
+import os
+
 import numpy as np
 import pytest
 import torch
 
 import oracle
-from parity import compare_quantize, to_np
+from parity import compare_quantize
 from paper_2606_07618_gb300 import workloads as W
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda"
-SAMPLE_ROWS = 48
 
 
 @pytest.fixture(scope="module")
@@ -42,63 +54,65 @@ def tensors_of(name):
     return wl, _cache[key]
 
 
-def sample_rows(rows):
-    idx = np.unique(np.concatenate([[0, rows - 1], np.linspace(0, rows - 1, SAMPLE_ROWS).astype(np.int64)]))
-    return idx
+def _threads():
+    return len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
 
 
 @pytest.mark.parametrize("name", W.ALL_CONFIGS)
-def test_workload_parity_full_size(B, name):
+def test_workload_parity_every_block(B, name, capsys):
+    from paper_2606_07618_gb300 import step as ST
     wl, ts = tensors_of(name)
-    obj = B.NVFP4_OBJ_WMSE if wl.objective == "wmse" else B.NVFP4_OBJ_MSE
+    wmse = wl.objective == "wmse"
+    obj = B.NVFP4_OBJ_WMSE if wmse else B.NVFP4_OBJ_MSE
     block = wl.block
-    win = (B.NVFP4_WINDOW_DEFAULT, B.NVFP4_WINDOW_DEFAULT)
-    for t, x, w in ts:
-        xd = x.to(DEV)
-        S = torch.empty(1, device=DEV)
-        st = torch.zeros(1, dtype=torch.int32, device=DEV)
-        ws = torch.empty(B.nvfp4_global_scale_workspace(xd.numel()), dtype=torch.uint8, device=DEV)
-        B.nvfp4_global_scale(xd, wl.fp8_div, S, st, ws)
+    xd = [x.to(DEV) for _, x, _ in ts]
+    wd = [w.to(DEV) for _, _, w in ts] if wmse else None
+    st = ST.for_workload(wl, xd, wd)
+    st()
+    torch.cuda.synchronize()
+    assert st.status.item() == 0
+    blocks = ties = 0
+    for i, (t, x, w) in enumerate(ts):
         xs = x.float().numpy()
         So, bad = oracle.global_scale(xs, wl.fp8_div)
-        assert S.item() == np.float32(So) and st.item() == 0 and not bad
-
+        assert st.S[i].item() == np.float32(So) and not bad, f"{t.name}: S"
         rows, cols = x.shape
-        out = B.empty_outputs(rows, cols, block, device=DEV, linear=True, swizzled=block == 16, loss=True)
-        wd = w.to(DEV) if obj == B.NVFP4_OBJ_WMSE else None
-        B.scalesweep_quantize(xd, block, S, obj, wd, 0, *win, out["codes"], out["sf_linear"], out["sf_swizzled"],
-                              out["block_loss"])
-        torch.cuda.synchronize()
+        o = st.outs[i]
+        wn = w.numpy() if wmse else None
+        ref = oracle.quantize(0, xs, block, So, obj, w=wn, w_row_stride=0, nthreads=_threads())
+        gpu = {"codes": o["codes"].cpu(), "sf_linear": o["sf_linear"].cpu(),
+               "sf_swizzled": o["sf_swizzled"].cpu() if o["sf_swizzled"] is not None else None}
+        stats = compare_quantize(xs, So, block, obj, w if wmse else None, 0, gpu, ref)
+        blocks += stats["blocks"]
+        ties += stats["near_tie_accepted"]
 
-        # sampled rows against the oracle (same S, same weights)
-        idx = sample_rows(rows)
-        sub = {"codes": out["codes"][idx], "sf_linear": out["sf_linear"][idx],
-               "block_loss": out["block_loss"].view(rows, -1)[idx].reshape(-1)}
-        wn = w.numpy() if obj == B.NVFP4_OBJ_WMSE else None
-        ref = oracle.quantize(0, xs[idx], block, So, obj, w=wn, w_row_stride=0)
-        compare_quantize(xs[idx], So, block, obj, wd, 0, sub, ref)
-
-        # properties of every block
-        sf = out["sf_linear"]
-        assert int(sf.max()) <= 126
-        if out["sf_swizzled"] is not None:
-            kb = cols // 16
-            r = torch.arange(rows, device=DEV).view(-1, 1)
-            k = torch.arange(kb, device=DEV).view(1, -1)
-            kpad4 = (kb + 3) // 4
-            off = ((r // 128) * kpad4 + k // 4) * 512 + (r % 32) * 16 + ((r // 32) % 4) * 4 + (k % 4)
-            assert torch.equal(out["sf_swizzled"][off.view(-1)].view(rows, kb), sf)
-        # reconstruction stays within half a grid step of the clipped value: |x_hat| <= 6 s S and finite
+        # dequantisation of the GPU's codes: bit-exact against the oracle's
         deq = torch.empty(rows, cols, device=DEV)
-        B.nvfp4_dequantize(out["codes"], sf, B.NVFP4_SF_LINEAR, S, rows, cols, block, deq)
-        vals = torch.from_numpy(np.array([oracle.e4m3_value(c) for c in range(127)] + [0.0] * 129,
-                                         dtype=np.float32)).to(DEV)
-        smax = (vals[sf.long()] * 6.0 * S).repeat_interleave(block, dim=1)
-        assert torch.isfinite(deq).all()
-        assert torch.all(deq.abs() <= smax * (1 + 1e-6))
-        # total loss of the tensor equals the sum of the per-block losses (x domain)
-        tot = float(((deq.double() - xd.double()) ** 2 * (wd.double() if wd is not None else 1.0)).sum())
-        est = float(out["block_loss"].double().sum()) * float(S.item()) ** 2
-        assert abs(tot - est) <= 1e-4 * est
-        del xd, out, deq, smax
-        torch.cuda.empty_cache()
+        if o["sf_swizzled"] is not None:
+            B.nvfp4_dequantize(o["codes"], o["sf_swizzled"], B.NVFP4_SF_SWIZZLED, st.S[i:i + 1], rows, cols, block,
+                               deq)
+        else:
+            B.nvfp4_dequantize(o["codes"], o["sf_linear"], B.NVFP4_SF_LINEAR, st.S[i:i + 1], rows, cols, block, deq)
+        torch.cuda.synchronize()
+        want = oracle.dequantize(gpu["codes"].numpy(), gpu["sf_linear"].numpy(), oracle.LAYOUT_LINEAR, So, rows,
+                                 cols, block)
+        assert np.array_equal(deq.cpu().numpy().view(np.uint32), want.view(np.uint32)), f"{t.name}: dequant"
+        del want
+
+        # summed loss: x-domain loss of the GPU's output vs the oracle's summed block optimum
+        err = (xd[i].double() - deq.double()) ** 2
+        if wmse:
+            err = err * wd[i].double()
+        tot_gpu = float(err.sum())
+        bl = ref["best"].copy()
+        if stats["near_tie_accepted"]:
+            d = np.nonzero(gpu["sf_linear"].numpy().reshape(-1) != ref["sf"].reshape(-1))[0]
+            bl[d] = oracle.block_losses_at(xs, block, So, gpu["sf_linear"].numpy(), obj, w=wn, w_row_stride=0,
+                                           nthreads=_threads())[d]
+        tot_ref = float(bl.sum()) * float(So) ** 2
+        assert abs(tot_gpu - tot_ref) <= 1e-5 * tot_ref, f"{t.name}: summed loss {tot_gpu} vs {tot_ref}"
+        del deq, err, ref
+    with capsys.disabled():
+        print(f"\n[parity] {name}: {blocks} blocks checked against the oracle, {ties} near-ties accepted")
+    del st, xd, wd
+    torch.cuda.empty_cache()

@@ -64,52 +64,61 @@ def make_group(dtype, obj, seed=0, shapes=SHAPES, row_weights=(3,)):
     return xs, ws, strides
 
 
-def run_group(B, xs, ws, strides, obj, D=256.0, S_in=None, ws_buf=None, status=None):
+def run_group(B, xs, ws, strides, obj, D=256.0, S_in=None, ws_buf=None, status=None, block=16, method=0):
     dev_x = [x.to(DEV) for x in xs]
     dev_w = [w.to(DEV) if w is not None else None for w in ws]
-    outs = [B.empty_outputs(x.shape[0], x.shape[1], 16, device=DEV, linear=True, swizzled=True) for x in xs]
+    outs = [B.empty_outputs(x.shape[0], x.shape[1], block, device=DEV, linear=True, swizzled=block == 16)
+            for x in xs]
     for o in outs:                                                   # poison: every byte must be written
-        o["codes"].fill_(0xEE)
-        o["sf_linear"].fill_(0xEE)
-        o["sf_swizzled"].fill_(0xEE)
+        for k in ("codes", "sf_linear", "sf_swizzled"):
+            if o[k] is not None:
+                o[k].fill_(0xEE)
     desc = B.group_descriptors(dev_x, dev_w, strides, [o["codes"] for o in outs], [o["sf_linear"] for o in outs],
                                [o["sf_swizzled"] for o in outs])
     dt = B.NVFP4_IN_BF16 if xs[0].dtype == torch.bfloat16 else B.NVFP4_IN_F32
     st = status if status is not None else torch.zeros(1, dtype=torch.int32, device=DEV)
+    call = (lambda d, S_, ws_: B.scalesweep_quantize_group(desc, dt, obj, d, S_, st, ws_, block=block)) \
+        if method == 0 else (lambda d, S_, ws_: B.absmax_quantize_group(desc, dt, d, S_, st, ws_, block=block))
     if S_in is None:
         S = torch.full((len(xs),), -1.0, device=DEV)
         if ws_buf is None:
             ws_buf = torch.empty(B.scalesweep_quantize_group_workspace(), dtype=torch.uint8, device=DEV)
-        B.scalesweep_quantize_group(desc, dt, obj, D, S, st, ws_buf)
+        call(D, S, ws_buf)
     else:
         S = S_in.clone()
-        B.scalesweep_quantize_group(desc, dt, obj, 0.0, S, st, None)
+        call(0.0, S, None)
     torch.cuda.synchronize()
     return S, st, outs, dev_x, dev_w
 
 
-def per_tensor(B, x, w, stride, obj, S=None, D=256.0):
+def per_tensor(B, x, w, stride, obj, S=None, D=256.0, block=16, method=0):
     st = torch.zeros(1, dtype=torch.int32, device=DEV)
     if S is None:
         S = torch.empty(1, device=DEV)
         wsb = torch.empty(B.nvfp4_global_scale_workspace(x.numel()), dtype=torch.uint8, device=DEV)
         B.nvfp4_global_scale(x, D, S, st, wsb)
-    o = B.empty_outputs(x.shape[0], x.shape[1], 16, device=DEV, linear=True, swizzled=True)
+    o = B.empty_outputs(x.shape[0], x.shape[1], block, device=DEV, linear=True, swizzled=block == 16)
     if x.numel():
-        B.scalesweep_quantize(x, 16, S, obj, w, stride, *WIN, o["codes"], o["sf_linear"], o["sf_swizzled"], None)
+        if method == 0:
+            B.scalesweep_quantize(x, block, S, obj, w, stride, *WIN, o["codes"], o["sf_linear"], o["sf_swizzled"],
+                                  None)
+        else:
+            B.absmax_quantize(x, block, S, o["codes"], o["sf_linear"], o["sf_swizzled"], None)
     torch.cuda.synchronize()
     return S, st, o
 
 
-def check_against_per_tensor(B, xs, ws, strides, obj, S, outs, dev_x, dev_w, static=False):
+def check_against_per_tensor(B, xs, ws, strides, obj, S, outs, dev_x, dev_w, static=False, block=16, method=0):
     for i, x in enumerate(dev_x):
-        S1, _, o1 = per_tensor(B, x, dev_w[i], strides[i], obj, S=S[i:i + 1] if static else None)
+        S1, _, o1 = per_tensor(B, x, dev_w[i], strides[i], obj, S=S[i:i + 1] if static else None, block=block,
+                               method=method)
         if not static:
             assert S[i].item() == S1.item(), f"tensor {i}: S {S[i].item()} vs {S1.item()}"
         if x.numel() == 0:
             continue
         for k in ("codes", "sf_linear", "sf_swizzled"):
-            assert torch.equal(outs[i][k], o1[k]), f"tensor {i}: {k}"
+            if o1[k] is not None:
+                assert torch.equal(outs[i][k], o1[k]), f"tensor {i}: {k}"
 
 
 @pytest.mark.parametrize("obj", [0, 1])
@@ -128,6 +137,39 @@ def test_group_dynamic_matches_oracle_and_per_tensor(B, dtype, obj):
         wn = ws[i].numpy() if ws[i] is not None else None
         ref = oracle.quantize(0, xs_np, 16, So, obj, w=wn, w_row_stride=strides[i])
         compare_quantize(xs_np, So, 16, obj, ws[i], strides[i], outs[i], ref)
+
+
+SHAPES64 = [(130, 192), (1, 64), (37, 128), (300, 512), (0, 64), (1000, 1024), (64, 320)]
+
+
+@pytest.mark.parametrize("dyn", [True, False])
+@pytest.mark.parametrize("block,obj,method", [(32, 0, 0), (32, 1, 0), (64, 0, 0), (64, 1, 0),
+                                              (16, 0, 1), (32, 0, 1), (64, 0, 1)])
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_group_blocks_and_absmax(B, dtype, block, obj, method, dyn):
+    """Blocks of 32 and 64 (two and four lanes per block) and the grouped AbsMax
+    launch: every tensor equals the oracle (near-tie rule) and, bit for bit,
+    the per-tensor call with the same scale."""
+    xs, ws, strides = make_group(dtype, obj, seed=7 + block + 3 * method, shapes=SHAPES64)
+    S_in = None
+    if not dyn:
+        S_in = torch.tensor([oracle.global_scale(x.float().numpy(), 256.0)[0] if x.numel() else 1.0 for x in xs],
+                            dtype=torch.float32, device=DEV)
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, obj, S_in=S_in, block=block, method=method)
+    assert st.item() == 0
+    check_against_per_tensor(B, xs, ws, strides, obj, S, outs, dev_x, dev_w, static=not dyn, block=block,
+                             method=method)
+    for i, x in enumerate(xs):
+        if x.numel() == 0:
+            continue
+        xs_np = x.float().numpy()
+        So = float(S[i].item())
+        if dyn:
+            assert So == np.float32(oracle.global_scale(xs_np, 256.0)[0]), f"tensor {i}"
+        wn = ws[i].numpy() if ws[i] is not None else None
+        ref = oracle.quantize(method, xs_np, block, So, obj if method == 0 else 0, w=wn if method == 0 else None,
+                              w_row_stride=strides[i])
+        compare_quantize(xs_np, So, block, obj, ws[i], strides[i], outs[i], ref, method=method)
 
 
 @pytest.mark.parametrize("obj", [0, 1])
