@@ -1,18 +1,22 @@
 #!/usr/bin/env python3
 """Benchmark of the NVFP4 ScaleSweep hot path on GB300.
 
-A step is one pass of the hot path over the Llama-3-8B-shaped layer (q, k, v,
-o, gate, up, down; 218.1M bf16 elements, synthetic N(0, 0.02^2) with 0.1%
-outlier input channels x20): the global scale S = amax/(6*256) of every tensor,
-then ScaleSweep with the WMSE objective (per-input-channel lognormal(0,1)
-weights), block 16, writing packed FP4 codes plus linear and swizzled E4M3
-scales.  The metric is Gelem/s of the whole step; the dominant kernel (the
-sweep) is also reported against its roofline.
+A step is one pass of the hot path over the largest single-GPU workload: two
+Qwen2.5-72B-shaped weights, 8192x29568 and 29568x8192 (484.4M bf16 elements,
+synthetic Laplace(0, 0.015) with 0.05% outlier input channels x30): the
+global scale S = amax/(6*256) of each matrix, then ScaleSweep with the WMSE
+objective (per-input-channel lognormal(0,1) weights), block 16, writing packed
+FP4 codes plus linear and swizzled E4M3 scales -- one grouped launch that
+reduces the scales while it sweeps.  The metric is Gelem/s of the whole step;
+the kernel is also reported against its FP32 and HBM rooflines.  Every other
+configuration (the 2048x2048 weight, the Llama-3-8B layer, the 8192x4096
+activation, K/V/Q, and the Qwen shapes at blocks 16/32/64 with MSE and WMSE) is
+timed as a leg in its own step's launch shape, beside AbsMax in the same shape.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl {gb300,reference}]
 
 With N > 1 the script runs under torch.distributed.run: every rank quantises its
-own copy of the layer (weak scaling, no collective on the data path); the
+own copy of the workload (weak scaling, no collective on the data path); the
 timed region is bracketed by barriers and the slowest rank's time is reported.
 """
 from __future__ import annotations
@@ -31,7 +35,10 @@ import torch
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-WORKLOAD = "llama8b"
+WORKLOAD = "qwen72b-b16-wmse"
+# every other configuration is timed as a leg in its own step's launch shape
+LEG_CONFIGS = ["qwen72b-b16-mse", "qwen72b-b32-mse", "qwen72b-b32-wmse", "qwen72b-b64-mse", "qwen72b-b64-wmse",
+               "weight-2048", "llama8b", "act-8192", "kvq"]
 METRIC = "NVFP4 ScaleSweep Gelem/s and % of GB300 HBM roofline; overhead vs AbsMax kernel"
 L2_BYTES = 129 * 1024 * 1024
 
@@ -123,14 +130,50 @@ class ClockSampler:
 
 
 # ----------------------------------------------------------------------------- workload
-def make_inputs(device: str):
+_inputs_cache: dict = {}
+
+
+def load_workload(name: str, device: str):
+    """Device copies of a workload's tensors and WMSE weights (drawn once per
+    distinct tensor set: the six Qwen2.5-72B-shaped configurations share it)."""
     from paper_2606_07618_gb300 import workloads as W
-    wl = W.workload(WORKLOAD)
-    xs, ws = [], []
-    for t in wl.tensors:
-        xs.append(W.draw(t).to(device))
-        ws.append(W.draw_weights(t).to(device))
+    wl = W.workload(name)
+    key = tuple((t.seed, t.rows, t.cols) for t in wl.tensors)
+    if key not in _inputs_cache:
+        _inputs_cache.clear()
+        torch.cuda.empty_cache()
+        _inputs_cache[key] = ([W.draw(t).to(device) for t in wl.tensors],
+                              [W.draw_weights(t).to(device) for t in wl.tensors])
+    xs, ws = _inputs_cache[key]
     return wl, xs, ws
+
+
+def make_inputs(device: str, name: str = "llama8b"):
+    wl, xs, ws = load_workload(name, device)
+    return wl, xs, ws
+
+
+def candidates(wl) -> int:
+    """Candidates per block of the default window (Sec. 4.2.2)."""
+    return 11 if (wl.objective == "mse" and wl.block == 16) else 16
+
+
+def alu_ops_per_elem(wl) -> int:
+    """Algorithmic FP32 work of the sweep per element: per candidate one
+    multiply (t = y r), one fma (e = y - q v), one fma accumulating e^2, and
+    for WMSE one more multiply (w e)."""
+    return (4 if wl.objective == "wmse" else 3) * candidates(wl)
+
+
+def hbm_bytes(wl, xs, both_layouts=True):
+    """Algorithmic HBM bytes of one step: the global-scale reduction reads each
+    input once, the sweep reads it again and writes the packed codes and the
+    scales (both layouts for block 16), plus the WMSE channel weights."""
+    inb = xs[0].element_size()
+    layouts = 2 if (both_layouts and wl.block == 16) else 1
+    per_elem = inb + inb + 0.5 + layouts / wl.block
+    wbytes = sum(4 * x.shape[1] for x in xs) if wl.objective == "wmse" else 0
+    return sum(x.numel() for x in xs) * per_elem + wbytes
 
 
 def traffic_per_launch(record, elems_per_launch):
@@ -174,54 +217,62 @@ def peaks():
         return 6800.0, "fallback"
 
 
+class L2Flush:
+    """Rewrites a buffer of twice the L2 size (on the timing stream) so that a
+    timed call that follows starts with nothing of its inputs in L2."""
+
+    def __init__(self, device):
+        self.buf = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
+
+    def __call__(self):
+        self.buf.fill_(1.0)
+
+
+def time_calls(fn, reps, stream, flush=None, warm=3):
+    """Mean device time of one call (CUDA events on `stream`), optionally with
+    L2 flushed before each call (then only the call is inside the events)."""
+    for _ in range(warm):
+        fn()
+    torch.cuda.synchronize()
+    if flush is None:
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    for a, b in ev:
+        flush()
+        a.record(stream)
+        fn()
+        b.record(stream)
+    torch.cuda.synchronize()
+    return sum(a.elapsed_time(b) for a, b in ev) / reps
+
+
 # ----------------------------------------------------------------------------- GPU arm
 def run_gpu(args, rank, world):
     from paper_2606_07618_gb300 import binding as B
+    from paper_2606_07618_gb300 import step as ST
     dev = f"cuda:{torch.cuda.current_device()}"
-    wl, xs, ws = make_inputs(dev)
-    n_el = [x.numel() for x in xs]
-    total = sum(n_el)
     stream = torch.cuda.current_stream()
-    S = torch.empty(len(xs), dtype=torch.float32, device=dev)
-    st = torch.zeros(1, dtype=torch.int32, device=dev)
-    wsp = torch.empty(B.nvfp4_global_scale_workspace(max(n_el)), dtype=torch.uint8, device=dev)
-    outs = [B.empty_outputs(x.shape[0], x.shape[1], 16, device=dev, linear=True, swizzled=True) for x in xs]
-    D = wl.fp8_div
-    win = (B.NVFP4_WINDOW_DEFAULT, B.NVFP4_WINDOW_DEFAULT)
+    wl, xs, ws = load_workload(WORKLOAD, dev)
+    total = sum(x.numel() for x in xs)
+    st = ST.for_workload(wl, xs, ws)
+    nsm = torch.cuda.get_device_properties(dev).multi_processor_count
+    hbm_peak, peak_kind = peaks()
 
-    def sweep(i):
-        o = outs[i]
-        B.scalesweep_quantize(xs[i], 16, S[i:i + 1], B.NVFP4_OBJ_WMSE, ws[i], 0, *win, o["codes"], o["sf_linear"],
-                              o["sf_swizzled"], None, stream=stream)
-
-    # The step: one grouped launch over the 7 tensors that also reduces every
-    # tensor's global scale (a ninth warp per CTA streams the reductions while
-    # the other eight sweep).  The same step as per-tensor launches is timed as
-    # a leg: global scales on a side stream, sweep i after amax i.
-    aux = torch.cuda.Stream()
-    wsps = [torch.empty_like(wsp) for _ in xs]
-    amax_done = [torch.cuda.Event() for _ in xs]
-    gws = torch.empty(B.scalesweep_quantize_group_workspace(), dtype=torch.uint8, device=dev)
-    desc = B.group_descriptors(xs, ws, [0] * len(xs), [o["codes"] for o in outs], [o["sf_linear"] for o in outs],
-                               [o["sf_swizzled"] for o in outs])
-
+    # The step: one grouped launch over both matrices that reduces each one's
+    # global scale in the same launch (a ninth warp per CTA streams the
+    # reductions while the other eight sweep) and sweeps every block.
     def step(events=None):
         if events is not None:
             events[0].record(stream)
-        B.scalesweep_quantize_group(desc, B.NVFP4_IN_BF16, B.NVFP4_OBJ_WMSE, D, S, st, gws, stream=stream)
+        st(stream=stream)
         if events is not None:
             events[1].record(stream)
-
-    def step_per_tensor():
-        aux.wait_stream(stream)
-        with torch.cuda.stream(aux):
-            for i, x in enumerate(xs):
-                B.nvfp4_global_scale(x, D, S[i:i + 1], st, wsps[i], stream=aux)
-                amax_done[i].record(aux)
-        for i in range(len(xs)):
-            stream.wait_event(amax_done[i])
-            sweep(i)
-        stream.wait_stream(aux)
 
     launches_per_step = 1   # the grouped kernel (the workspace reset is a memset; these shapes need no pad kernel)
 
@@ -242,204 +293,217 @@ def run_gpu(args, rank, world):
     if world > 1:
         torch.distributed.barrier()
     ms = t0.elapsed_time(t1)
-    sweep_ms = sum(ev[k][0].elapsed_time(ev[k][1]) for k in range(args.steps))
+    kern_ms = sum(ev[k][0].elapsed_time(ev[k][1]) for k in range(args.steps)) / args.steps
     ms = reduce_max_ms(ms, world, dev)
     ms_step = ms / args.steps
     value = world * total / (ms_step * 1e-3) / 1e9
+    assert int(st.status.item()) == 0, "non-finite input detected"
 
-    # status word: any non-finite input would have been flagged
-    assert int(st.item()) == 0, "non-finite input detected"
-
-    # ---- roofline of the dominant (only) kernel, the grouped launch, from the events above
-    # algorithmic bytes: the global-scale reduction reads each input once, the
-    # sweep reads it again and writes codes and both scale layouts; plus the
-    # channel weights
-    bpe = alg_bytes_per_elem() + 2
-    alg_bytes = sum(n * bpe + 4 * x.shape[1] for n, x in zip(n_el, xs))
-    sweep_s_per_step = sweep_ms / args.steps * 1e-3
-    gbs = alg_bytes / sweep_s_per_step / 1e9
-    hbm_peak, peak_kind = peaks()
+    # ---- roofline of the dominant (only) kernel, from the per-step events
     clk_sum = clk.summary()
     sm_mhz = clk_sum["sm_mhz"] or clk_sum["sm_max_mhz"] or 2070
-    nsm = torch.cuda.get_device_properties(dev).multi_processor_count
-    # algorithmic FP32 work of the WMSE sweep: per element and candidate one
-    # multiply (t = y r), one fma (e = y - q v), one multiply (w e) and one fma
-    # (accumulate); 16 candidates per block ([-8, 7]).
-    ops = 4 * 16 * total
     alu_peak = nsm * 128 * sm_mhz * 1e6
-    alu_achieved = ops / sweep_s_per_step
-    roofline = {"bound": "alu", "achieved": round(alu_achieved / 1e12, 3), "peak": round(alu_peak / 1e12, 3),
-                "unit": "Tops/s", "frac": round(alu_achieved / alu_peak, 4), "traffic": None,
-                "kernel": "quantize_group_kernel<bf16,WMSE,dynamic S> (7 tensors, one launch per step)",
-                "peak_note": f"{nsm} SMs x 128 FP32 lanes x median SM clock {sm_mhz} MHz",
-                "hbm": {"achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s", "frac": round(gbs / hbm_peak, 4),
-                        "peak_kind": peak_kind, "bytes_per_elem": bpe},
-                "launch_ms": round(sweep_s_per_step * 1e3, 4),
+
+    def fracs(wl_, xs_, t_ms):
+        n = sum(x.numel() for x in xs_)
+        gbs = hbm_bytes(wl_, xs_) / (t_ms * 1e-3) / 1e9
+        ops = alu_ops_per_elem(wl_) * n / (t_ms * 1e-3)
+        return round(gbs, 1), round(gbs / hbm_peak, 4), round(ops / 1e12, 3), round(ops / alu_peak, 4)
+
+    gbs, hfrac, tops, afrac = fracs(wl, xs, kern_ms)
+    roofline = {"bound": "alu", "achieved": tops, "peak": round(alu_peak / 1e12, 3), "unit": "Tops/s",
+                "frac": afrac, "traffic": None,
+                "kernel": f"quantize_group_kernel<bf16,ScaleSweep,WMSE,block {wl.block},dynamic S> "
+                          f"({len(xs)} tensors, one launch per step)",
+                "peak_note": f"{nsm} SMs x 128 FP32 lanes x median SM clock {sm_mhz} MHz "
+                             f"(of measured clock; the work is {alu_ops_per_elem(wl)} FP32 ops per element: "
+                             f"{candidates(wl)} candidates x 4)",
+                "hbm": {"achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": hfrac, "peak_kind": peak_kind,
+                        "bytes": round(hbm_bytes(wl, xs)), "bytes_per_elem": round(hbm_bytes(wl, xs) / total, 4)},
+                "launch_ms": round(kern_ms, 4),
                 "launch_note": "events around the call: the 256-byte workspace memset and the kernel"}
-    roofline["traffic"] = traffic_per_launch("quantize_group_kernel_wmse_traffic.json", total)
+    roofline["traffic"] = traffic_per_launch("quantize_group_kernel_qwen72b_traffic.json", total)
 
-    # ---- overhead vs the AbsMax kernel on the same tensors, same S and layouts
-    def time_leg(fn, reps):
-        for _ in range(3):
-            fn()
-        torch.cuda.synchronize()
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        for _ in range(reps):
-            fn()
-        b.record(stream)
-        torch.cuda.synchronize()
-        return a.elapsed_time(b) / reps
+    reps = max(3, min(20, args.steps))
+    flush = L2Flush(dev)
+    legs = {}
 
-    def absmax_all():
+    # ---- every configuration in its step's launch shape, and AbsMax in the same shape
+    for name in ([] if args.no_legs else LEG_CONFIGS):
+        wl_c, xs_c, ws_c = load_workload(name, dev)
+        sc = ST.for_workload(wl_c, xs_c, ws_c)
+        small = sum(x.numel() * x.element_size() for x in xs_c) < 2 * L2_BYTES
+        fl = flush if small else None
+        t_ss = time_calls(lambda: sc(stream=stream), reps, stream, fl)
+        t_ab = time_calls(lambda: sc.absmax(stream=stream), reps, stream, fl)
+        assert int(sc.status.item()) == 0
+        n = sc.numel
+        g, hf, tp, af = fracs(wl_c, xs_c, t_ss)
+        legs[name] = {"elements": n, "launch": "fused dynamic" if sc.fused else f"grouped dynamic x{len(xs_c)}",
+                      "block": wl_c.block, "objective": wl_c.objective, "D": wl_c.fp8_div, "ms": round(t_ss, 4),
+                      "gelem_s": round(n / (t_ss * 1e-3) / 1e9, 2), "hbm_gbs": g, "hbm_frac": hf,
+                      "fp32_tops": tp, "fp32_frac": af, "absmax_ms": round(t_ab, 4),
+                      "overhead_vs_absmax": round(t_ss / t_ab, 3), "l2": "flushed before each call" if small
+                      else "inputs > L2"}
+        del sc
+    _inputs_cache.clear()                       # the headline's tensors stay referenced by xs / ws
+
+    # ---- the headline workload's other legs
+    def gel(t):
+        return round(total / (t * 1e-3) / 1e9, 2)
+
+    st_static = ST.QuantizeStep(xs, ws, block=wl.block, objective=B.NVFP4_OBJ_WMSE, fp8_div=wl.fp8_div)
+    st_static(stream=stream)
+    S_fixed = st_static.S.clone()
+
+    def static_sweep():
+        B.scalesweep_quantize_group(st_static.desc, st_static.dtype, B.NVFP4_OBJ_WMSE, 0.0, S_fixed, None, None,
+                                    stream=stream, block=wl.block)
+
+    def absmax_static():
+        B.absmax_quantize_group(st_static.desc, st_static.dtype, 0.0, S_fixed, None, None, stream=stream,
+                                block=wl.block)
+
+    gsw = [torch.empty(B.nvfp4_global_scale_workspace(x.numel()), dtype=torch.uint8, device=dev) for x in xs]
+    Sg = torch.empty(len(xs), device=dev)
+    win = (B.NVFP4_WINDOW_DEFAULT, B.NVFP4_WINDOW_DEFAULT)
+
+    def per_tensor_launches():
         for i, x in enumerate(xs):
-            o = outs[i]
-            B.absmax_quantize(x, 16, S[i:i + 1], o["codes"], o["sf_linear"], o["sf_swizzled"], None, stream=stream)
+            o = st_static.outs[i]
+            B.nvfp4_global_scale(x, wl.fp8_div, Sg[i:i + 1], None, gsw[i], stream=stream)
+            B.scalesweep_quantize(x, wl.block, Sg[i:i + 1], B.NVFP4_OBJ_WMSE, ws[i], 0, *win, o["codes"],
+                                  o["sf_linear"], o["sf_swizzled"], None, stream=stream)
 
-    def sweep_all():
-        for i in range(len(xs)):
-            sweep(i)
-
-    def sweep_mse_all():
+    def four_six():
         for i, x in enumerate(xs):
-            o = outs[i]
-            B.scalesweep_quantize(x, 16, S[i:i + 1], B.NVFP4_OBJ_MSE, None, 0, *win, o["codes"], o["sf_linear"],
-                                  o["sf_swizzled"], None, stream=stream)
+            o = st_static.outs[i]
+            B.four_over_six_quantize(x, wl.block, S_fixed[i:i + 1], B.NVFP4_OBJ_WMSE, ws[i], 0, o["codes"],
+                                     o["sf_linear"], o["sf_swizzled"], None, stream=stream)
 
-    def four_six_all():
+    dq = torch.empty(max(x.numel() for x in xs), dtype=torch.bfloat16, device=dev)
+
+    def dequant():
         for i, x in enumerate(xs):
-            o = outs[i]
-            B.four_over_six_quantize(x, 16, S[i:i + 1], B.NVFP4_OBJ_WMSE, ws[i], 0, o["codes"], o["sf_linear"],
-                                     o["sf_swizzled"], None, stream=stream)
+            o = st_static.outs[i]
+            B.nvfp4_dequantize(o["codes"], o["sf_swizzled"], B.NVFP4_SF_SWIZZLED, S_fixed[i:i + 1], x.shape[0],
+                               x.shape[1], wl.block, dq[:x.numel()], stream=stream)
 
-    dq = torch.empty(max(n_el), dtype=torch.bfloat16, device=dev)
-
-    def dequant_all():
+    def global_scales():
         for i, x in enumerate(xs):
-            o = outs[i]
-            B.nvfp4_dequantize(o["codes"], o["sf_swizzled"], B.NVFP4_SF_SWIZZLED, S[i:i + 1], x.shape[0], x.shape[1],
-                               16, dq[:x.numel()], stream=stream)
+            B.nvfp4_global_scale(x, wl.fp8_div, Sg[i:i + 1], None, gsw[i], stream=stream)
 
-    def amax_all():
-        for i, x in enumerate(xs):
-            B.nvfp4_global_scale(x, D, S[i:i + 1], st, wsp, stream=stream)
+    if args.no_legs:
+        return dict(value=value, ms_step=ms_step, total=total, roofline=roofline, clocks=clk_sum, legs=None,
+                    overhead=None, e2e=None, cpu=None, launches=launches_per_step * args.steps, wl=wl)
+    t_gs = time_calls(static_sweep, reps, stream)
+    t_as = time_calls(absmax_static, reps, stream)
+    t_pt = time_calls(per_tensor_launches, reps, stream)
+    t_46 = time_calls(four_six, reps, stream)
+    t_dq = time_calls(dequant, reps, stream)
+    t_am = time_calls(global_scales, reps, stream)
+    t_ab = legs[WORKLOAD]["absmax_ms"] if WORKLOAD in legs else time_calls(lambda: st.absmax(stream=stream), reps,
+                                                                             stream)
+    legs[WORKLOAD + " (headline) static scales"] = {
+        "scalesweep_grouped_static": {"ms": round(t_gs, 4), "gelem_s": gel(t_gs)},
+        "absmax_grouped_static": {"ms": round(t_as, 4), "gelem_s": gel(t_as)},
+        "per_tensor_global_scale_then_sweep": {"ms": round(t_pt, 4), "gelem_s": gel(t_pt)},
+        "four_over_six_wmse_per_tensor": {"ms": round(t_46, 4), "gelem_s": gel(t_46)},
+        "dequant_bf16_swizzled": {"ms": round(t_dq, 4), "gelem_s": gel(t_dq)},
+        "global_scale_per_tensor": {"ms": round(t_am, 4), "gelem_s": gel(t_am)}}
+    overhead = {"scalesweep_wmse_vs_absmax_grouped_dynamic": round(kern_ms / t_ab, 3),
+                "scalesweep_wmse_vs_absmax_grouped_static": round(t_gs / t_as, 3),
+                "per_config": {k: v["overhead_vs_absmax"] for k, v in legs.items() if "overhead_vs_absmax" in v}}
 
-    def sweep_group_static():
-        B.scalesweep_quantize_group(desc, B.NVFP4_IN_BF16, B.NVFP4_OBJ_WMSE, 0.0, S, st, None, stream=stream)
-
-    reps = max(3, min(50, args.steps))
-    t_pt = time_leg(step_per_tensor, reps)
-    t_gs = time_leg(sweep_group_static, reps)
-    t_abs = time_leg(absmax_all, reps)
-    t_ss = time_leg(sweep_all, reps)
-    t_ssm = time_leg(sweep_mse_all, reps)
-    t_46 = time_leg(four_six_all, reps)
-    t_dq = time_leg(dequant_all, reps)
-    t_am = time_leg(amax_all, reps)
-    gel = lambda ms_: round(total / (ms_ * 1e-3) / 1e9, 2)
-    legs = {"step_per_tensor_launches": {"ms": round(t_pt, 4), "gelem_s": gel(t_pt)},
-            "scalesweep_wmse_grouped_static_scales": {"ms": round(t_gs, 4), "gelem_s": gel(t_gs)},
-            "scalesweep_wmse": {"ms": round(t_ss, 4), "gelem_s": gel(t_ss)},
-            "scalesweep_mse": {"ms": round(t_ssm, 4), "gelem_s": gel(t_ssm)},
-            "absmax": {"ms": round(t_abs, 4), "gelem_s": gel(t_abs)},
-            "four_over_six_wmse": {"ms": round(t_46, 4), "gelem_s": gel(t_46)},
-            "dequant_bf16": {"ms": round(t_dq, 4), "gelem_s": gel(t_dq)},
-            "global_scale": {"ms": round(t_am, 4), "gelem_s": gel(t_am)}}
-    overhead = {"scalesweep_wmse_vs_absmax": round(t_ss / t_abs, 3), "scalesweep_mse_vs_absmax": round(t_ssm / t_abs, 3)}
-
-    # ---- end to end through the public API with host buffers
+    # ---- end to end through the public API (QuantizeStep) with host buffers
     e2e = None
     if not args.no_e2e:
-        hx = [x.cpu().pin_memory() for x in xs]
-        hcodes = [torch.empty_like(o["codes"], device="cpu").pin_memory() for o in outs]
-        hsfl = [torch.empty_like(o["sf_linear"], device="cpu").pin_memory() for o in outs]
-        hsfs = [torch.empty_like(o["sf_swizzled"], device="cpu").pin_memory() for o in outs]
-        # two sets of device buffers, alternating between steps: the upload of
-        # step k+1 only waits for the kernels of step k-1, so the host link
-        # (the bound here) never idles between steps
-        dx = [[torch.empty_like(x) for x in xs] for _ in range(2)]
-        eouts = [[B.empty_outputs(x.shape[0], x.shape[1], 16, device=dev, linear=True, swizzled=True) for x in xs]
-                 for _ in range(2)]
-        up, down = torch.cuda.Stream(), torch.cuda.Stream()
-        S2 = torch.empty(len(xs), dtype=torch.float32, device=dev)
-        wsp2 = torch.empty_like(wsp)
-        comp_done = [torch.cuda.Event(), torch.cuda.Event()]
-        d2h_done = [torch.cuda.Event(), torch.cuda.Event()]
-        state = {"k": 0}
-
-        def e2e_step():
-            # H2D on `up`, kernels on `stream`, D2H on `down`; events order each
-            # tensor's copy -> compute -> copy; buffer set k % 2
-            pb = state["k"] & 1
-            first_use = state["k"] < 2
-            state["k"] += 1
-            loaded, done = [], []
-            if not first_use:
-                up.wait_event(comp_done[pb])        # step k-2's kernels are done with dx[pb]
-            for i in range(len(xs)):
-                with torch.cuda.stream(up):
-                    dx[pb][i].copy_(hx[i], non_blocking=True)
-                    ev = torch.cuda.Event()
-                    ev.record(up)
-                    loaded.append(ev)
-            if not first_use:
-                stream.wait_event(d2h_done[pb])     # step k-2's downloads are done with eouts[pb]
-            for i in range(len(xs)):
-                stream.wait_event(loaded[i])
-                o = eouts[pb][i]
-                B.nvfp4_global_scale(dx[pb][i], D, S2[i:i + 1], st, wsp2, stream=stream)
-                B.scalesweep_quantize(dx[pb][i], 16, S2[i:i + 1], B.NVFP4_OBJ_WMSE, ws[i], 0, *win, o["codes"],
-                                      o["sf_linear"], o["sf_swizzled"], None, stream=stream)
-                ev = torch.cuda.Event()
-                ev.record(stream)
-                done.append(ev)
-            comp_done[pb].record(stream)
-            with torch.cuda.stream(down):
-                for i in range(len(xs)):
-                    down.wait_event(done[i])
-                    o = eouts[pb][i]
-                    hcodes[i].copy_(o["codes"], non_blocking=True)
-                    hsfl[i].copy_(o["sf_linear"], non_blocking=True)
-                    hsfs[i].copy_(o["sf_swizzled"], non_blocking=True)
-            d2h_done[pb].record(down)
-
-        def e2e_time(reps):
-            for _ in range(3):
-                e2e_step()
-            torch.cuda.synchronize()
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a.record(stream)
-            up.wait_stream(stream)
-            for _ in range(reps):
-                e2e_step()
-            stream.wait_stream(up)
-            stream.wait_stream(down)                # the last step's results are on the host
-            b.record(stream)
-            torch.cuda.synchronize()
-            return a.elapsed_time(b) / reps
-
-        e_reps = max(3, min(20, args.steps))
-        t_e2e = e2e_time(e_reps)
-        h2d = sum(x.numel() * x.element_size() for x in xs)
-        d2h = sum(o["codes"].numel() + o["sf_linear"].numel() + o["sf_swizzled"].numel() for o in outs)
-
-        def h2d_only():
-            for i in range(len(xs)):
-                dx[0][i].copy_(hx[i], non_blocking=True)
-
-        t_h2d = time_leg(h2d_only, e_reps)
-        e2e = {"value": round(world * total / (t_e2e * 1e-3) / 1e9, 3), "unit": "Gelem/s",
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(t_e2e, 4),
-               "h2d_gb_s_alone": round(h2d / (t_h2d * 1e-3) / 1e9, 1),
-               "streams": "H2D, compute and D2H on three streams, event-ordered per tensor, two buffer sets"}
+        e2e = run_e2e(wl, xs, ws, dev, stream, world, args)
 
     # ---- CPU baseline: the oracle on a bounded sample, rank 0 at N = 1 only
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        cpu = cpu_baseline(wl, [x.cpu() for x in xs], [w.cpu() for w in ws], S.cpu(), budget_s=args.cpu_seconds)
+        cpu = cpu_baseline(wl, [x.cpu() for x in xs], [w.cpu() for w in ws], st.S.cpu(), budget_s=args.cpu_seconds)
 
     return dict(value=value, ms_step=ms_step, total=total, roofline=roofline, clocks=clk_sum, legs=legs,
                 overhead=overhead, e2e=e2e, cpu=cpu, launches=launches_per_step * args.steps, wl=wl)
+
+
+def run_e2e(wl, xs, ws, dev, stream, world, args):
+    """The step through the public API with pinned host buffers: every step
+    uploads its inputs, quantises them (one QuantizeStep call) and downloads
+    codes and both scale layouts.  H2D, compute and D2H run on three streams,
+    event-ordered per step, with two device buffer sets alternating so the
+    upload of step k+1 only waits for the kernels of step k-1."""
+    from paper_2606_07618_gb300 import step as ST
+    hx = [x.cpu().pin_memory() for x in xs]
+    sets = []
+    for _ in range(2):
+        dx = [torch.empty_like(x) for x in xs]
+        sets.append((dx, ST.for_workload(wl, dx, ws)))
+    hout = [{k: torch.empty_like(v, device="cpu").pin_memory() for k, v in o.items() if v is not None}
+            for o in sets[0][1].outs]
+    up, down = torch.cuda.Stream(), torch.cuda.Stream()
+    comp_done = [torch.cuda.Event(), torch.cuda.Event()]
+    d2h_done = [torch.cuda.Event(), torch.cuda.Event()]
+    state = {"k": 0}
+
+    def e2e_step():
+        pb = state["k"] & 1
+        first_use = state["k"] < 2
+        state["k"] += 1
+        dx, sc = sets[pb]
+        if not first_use:
+            up.wait_event(comp_done[pb])            # step k-2's kernels are done with this input set
+        with torch.cuda.stream(up):
+            for i in range(len(xs)):
+                dx[i].copy_(hx[i], non_blocking=True)
+        loaded = torch.cuda.Event()
+        loaded.record(up)
+        if not first_use:
+            stream.wait_event(d2h_done[pb])         # step k-2's downloads are done with these outputs
+        stream.wait_event(loaded)
+        sc(stream=stream)
+        comp_done[pb].record(stream)
+        with torch.cuda.stream(down):
+            down.wait_event(comp_done[pb])
+            for i, o in enumerate(sc.outs):
+                for k, h in hout[i].items():
+                    h.copy_(o[k], non_blocking=True)
+        d2h_done[pb].record(down)
+
+    def e2e_time(reps):
+        for _ in range(3):
+            e2e_step()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        up.wait_stream(stream)
+        for _ in range(reps):
+            e2e_step()
+        stream.wait_stream(up)
+        stream.wait_stream(down)                    # the last step's results are on the host
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps
+
+    e_reps = max(3, min(10, args.steps))
+    t_e2e = e2e_time(e_reps)
+    total = sum(x.numel() for x in xs)
+    h2d = sum(x.numel() * x.element_size() for x in xs)
+    d2h = sum(h.numel() * h.element_size() for d in hout for h in d.values())
+    dx0 = sets[0][0]
+
+    def h2d_only():
+        for i in range(len(xs)):
+            dx0[i].copy_(hx[i], non_blocking=True)
+
+    t_h2d = time_calls(h2d_only, e_reps, stream)
+    return {"value": round(world * total / (t_e2e * 1e-3) / 1e9, 3), "unit": "Gelem/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(t_e2e, 4),
+            "h2d_gb_s_alone": round(h2d / (t_h2d * 1e-3) / 1e9, 1),
+            "link_bound_gelem_s": round(total / (t_h2d * 1e-3) / 1e9, 2),
+            "streams": "H2D, compute and D2H on three streams, event-ordered per step, two buffer sets"}
 
 
 def cpu_baseline(wl, xs_cpu, ws_cpu, S_cpu, budget_s=12.0, probe_rows=64):
@@ -448,6 +512,7 @@ def cpu_baseline(wl, xs_cpu, ws_cpu, S_cpu, budget_s=12.0, probe_rows=64):
     import oracle
     oracle.build()
     threads = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    obj = oracle.WMSE if wl.objective == "wmse" else oracle.MSE
 
     def run(rows):
         t = time.perf_counter()
@@ -456,8 +521,8 @@ def cpu_baseline(wl, xs_cpu, ws_cpu, S_cpu, budget_s=12.0, probe_rows=64):
             r = min(rows, x.shape[0])
             xs = x[:r].float().numpy()
             S = float(S_cpu[i]) if S_cpu is not None else oracle.global_scale(xs, wl.fp8_div)[0]
-            oracle.quantize(0, xs, wl.block, S, oracle.WMSE if wl.objective == "wmse" else oracle.MSE,
-                            w=ws_cpu[i].numpy(), w_row_stride=0, nthreads=threads)
+            oracle.quantize(0, xs, wl.block, S, obj, w=ws_cpu[i].numpy() if obj == oracle.WMSE else None,
+                            w_row_stride=0, nthreads=threads)
             n += xs.size
         return n, time.perf_counter() - t
 
@@ -468,7 +533,7 @@ def cpu_baseline(wl, xs_cpu, ws_cpu, S_cpu, budget_s=12.0, probe_rows=64):
     n, dt = run(rows)
     return {"value": round(n / dt / 1e9, 6), "unit": "Gelem/s", "cores": threads, "kind": "oracle",
             "sample": f"first {rows} rows of each of the {len(xs_cpu)} {wl.name} tensors ({n} elements, "
-                      f"{dt:.1f} s), same S, WMSE, block {wl.block}"}
+                      f"{dt:.1f} s), same S, {wl.objective.upper()}, block {wl.block}"}
 
 
 # ----------------------------------------------------------------------------- reference arm
@@ -484,12 +549,13 @@ def run_reference(args, rank, world):
     ws = [W.draw_weights(t) for t in wl.tensors]
     threads = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
     xf = [x.float().numpy() for x in xs]
-    # S of each full tensor would need the whole tensor; the sample's own amax is used
-    Ss = [oracle.global_scale(x, wl.fp8_div)[0] for x in xf]
+    obj = oracle.WMSE if wl.objective == "wmse" else oracle.MSE
 
     def step():
-        for x, w, S in zip(xf, ws, Ss):
-            oracle.quantize(0, x, wl.block, S, oracle.WMSE, w=w.numpy(), w_row_stride=0, nthreads=threads)
+        for x, w in zip(xf, ws):
+            # the per-call global scale of the sample, then the sweep
+            S = oracle.global_scale(x, wl.fp8_div)[0]
+            oracle.quantize(0, x, wl.block, S, obj, w=w.numpy(), w_row_stride=0, nthreads=threads)
 
     for _ in range(args.warmup):
         step()
@@ -505,18 +571,20 @@ def run_reference(args, rank, world):
             "config": config_dict(wl, world),
             "cpu_baseline": {"value": round(value, 6), "unit": "Gelem/s", "cores": threads, "kind": "oracle",
                              "sample": f"first {rows} rows of each of the {len(xf)} {wl.name} tensors per step ({n} "
-                                       f"elements), WMSE, block 16, S from the sample"},
+                                       f"elements): global scale of the sample, then the sweep, "
+                                       f"{wl.objective.upper()}, block {wl.block}"},
             "e2e": {"value": round(value, 6), "unit": "Gelem/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
 def config_dict(wl, world):
-    return {"workload": "llama3-8b-layer-weights-wmse", "tensors": {t.name: [t.rows, t.cols] for t in wl.tensors},
+    return {"workload": "qwen2.5-72b-shaped-weights-wmse-block16",
+            "tensors": {t.name: [t.rows, t.cols] for t in wl.tensors},
             "elements": wl.numel, "input": "bf16", "block": wl.block, "objective": wl.objective,
-            "global_scale": f"amax/(6*{int(wl.fp8_div)}) computed every step", "scale_layouts": "linear+swizzled",
+            "global_scale": f"amax/(6*{int(wl.fp8_div)}) computed every step, in the launch",
+            "scale_layouts": "linear+swizzled",
             "parallelism": f"replicas{world}" if world > 1 else "single-gpu",
-            "l2": "no flush: each step streams the 436 MB of inputs (> 129 MB L2) twice, once for the global scales "
-                  "and once for the sweep; inside the one launch tensor i+1's scale is reduced while tensor i is "
-                  "swept"}
+            "l2": "no flush: each step streams the 968 MB of inputs (> 129 MB L2) twice, once for the global scales "
+                  "and once for the sweep; inside the one launch matrix 2's scale is reduced while matrix 1 is swept"}
 
 
 def run_kernel_case(args):
@@ -564,7 +632,23 @@ def run_kernel_case(args):
     d1 = B.group_descriptors([x], [w], [0], [o["codes"]], [o["sf_linear"]], [o["sf_swizzled"]])
     fns["sweep_wmse_group"] = lambda: B.scalesweep_quantize_group(d1, B.NVFP4_IN_BF16, 1, 0.0, S, None, None)
     fns["wmse_group_dynamic"] = lambda: B.scalesweep_quantize_group(d1, B.NVFP4_IN_BF16, 1, 256.0, S1, None, gws)
-    if args.kernel_case.startswith(("group_layer", "layer_")):
+    if args.kernel_case.startswith("qwen"):
+        # the headline step (both Qwen2.5-72B-shaped matrices, WMSE, in-launch
+        # scales), or a slice of each (2048 and 7392 leading rows: 242 MB of
+        # inputs, still above L2) for profiler captures
+        from paper_2606_07618_gb300 import step as ST
+        wlq, qx, qw = load_workload(WORKLOAD, dev)
+        if args.kernel_case.startswith("qwen_slice"):
+            qx = [qx[0][:2048], qx[1][:7392]]
+        sq = ST.for_workload(wlq, qx, qw)
+        fns["qwen_group"] = fns["qwen_slice_group"] = lambda: sq()
+        fns["qwen_absmax_group"] = fns["qwen_slice_absmax_group"] = lambda: sq.absmax()
+        sq()
+        Sq = sq.S.clone()
+        fns["qwen_group_static"] = fns["qwen_slice_group_static"] = lambda: B.scalesweep_quantize_group(
+            sq.desc, B.NVFP4_IN_BF16, 1, 0.0, Sq, None, None, block=wlq.block)
+        n = sq.numel
+    elif args.kernel_case.startswith(("group_layer", "layer_")):
         # the Llama-3-8B layer in one grouped launch (dynamic scales), as the bench step
         _, xs, wl_ws = make_inputs(dev)
         lo = [B.empty_outputs(t.shape[0], t.shape[1], 16, device=dev, linear=True, swizzled=True) for t in xs]
@@ -856,10 +940,11 @@ def run_ldlq(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-legs", action="store_true", help="time the headline step only (profiler launch lists)")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-rows", type=int, default=64)
@@ -868,7 +953,8 @@ def main():
                              "sweep_wmse_group", "wmse_group_dynamic", "group_layer", "group_layer_static",
                              "sweep_wmse_tight", "sweep_mse_tight",
                              "layer_per_tensor_static", "group_layer_linear", "group_layer_static_linear",
-                             "mse_fused", "wmse_fused"])
+                             "mse_fused", "wmse_fused", "qwen_group", "qwen_group_static", "qwen_absmax_group",
+                             "qwen_slice_group", "qwen_slice_group_static", "qwen_slice_absmax_group"])
     ap.add_argument("--rows", type=int, default=16384)
     ap.add_argument("--cols", type=int, default=8192)
     ap.add_argument("--block", type=int, default=16)
@@ -913,7 +999,8 @@ def main():
         out = {"metric": METRIC, "value": round(r["value"], 3), "unit": "Gelem/s", "n_gpus": world,
                "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(r["ms_step"], 4),
                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-               "data": "synthetic (seeded N(0,0.02^2) Llama-3-8B-shaped weights, lognormal channel weights)",
+               "data": "synthetic (seeded Laplace(0,0.015) Qwen2.5-72B-shaped weights with x30 outlier channels, "
+                       "lognormal channel weights)",
                "config": config_dict(wl, world), "roofline": r["roofline"], "clocks": r["clocks"],
                "gpu_launches": r["launches"], "legs": r["legs"], "overhead_vs_absmax": r["overhead"],
                "e2e": r["e2e"], "cpu_baseline": r["cpu"]}

@@ -223,13 +223,13 @@ size_t scalesweep_quantize_group_workspace(void);
  *   fp8_div     0: static global scales, S[i] is read for tensor i.
  *               > 0: per-call (dynamic) global scales, S[i] = fl32(amax_i /
  *               fl32(6*fp8_div)) over tensor i (Sec. 4.2.1) is computed in the
- *               same launch and written; tensor i's reduction overlaps the sweep
- *               of the smaller tensors before it (cooperative launch, preceded
- *               by a cudaMemsetAsync of the workspace counters).
+ *               same launch and written: every warp first reduces its share of
+ *               every tensor, then a grid barrier, then the sweep (cooperative
+ *               launch, preceded by a cudaMemsetAsync of the workspace counters).
  *   S           device float[count].
  *   status_dev  optional device int: bit 0 OR-ed in for NaN/inf input (dynamic
- *               only), bit 1 if a wait for a scale timed out (about a second per
- *               wait; outputs are then incomplete -- a resident grid makes this
+ *               only), bit 1 if the grid barrier timed out (about a second; no
+ *               outputs are written then -- a resident grid makes this
  *               unreachable in practice).
  *   workspace   scalesweep_quantize_group_workspace() bytes, 16-byte aligned, no
  *               initialisation (dynamic only; may be NULL for static scales).

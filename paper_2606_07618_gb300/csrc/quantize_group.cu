@@ -5,13 +5,11 @@
 //
 // Why: a transformer layer has tensors of very different sizes (k/v are 1/14
 // of gate/up/down in Llama-3-8B).  One launch per tensor pays a ramp-down tail
-// per launch, and the HBM-bound amax pass of each tensor either runs before
-// its ALU-bound sweep or competes with it from a second stream.  Here the
-// segments of all tensors form one concatenated index space walked by one
-// grid-stride loop (a single tail), and the amax reductions run beside the
-// sweep inside the same launch.
+// per launch and, with per-call scales, a separate amax launch per tensor.
+// Here the segments of all tensors form one concatenated index space walked
+// by one grid-stride loop (a single tail).
 //
-// Sweep warps (8 per CTA).  A CTA walks 256 consecutive segments per
+// Sweep (8 warps per CTA).  A CTA walks 256 consecutive segments per
 // iteration; every tensor's segment range is padded to a multiple of 256, so
 // the tensor index t is CTA-uniform and the descriptor fields are read as
 // uniform kernel-parameter operands.  The per-segment sweep is the one of
@@ -20,19 +18,21 @@
 // and both scale layouts; blocks of 32/64 are 2/4 lanes combined by
 // xor-shuffles (a CTA's 256 segments always hold whole blocks).
 //
-// Reduction warp (a ninth warp per CTA, dynamic scales only).  The reduction
-// warps of the grid split every tensor's 16-byte input vectors round-robin
-// (vector aw*32 + lane + j*NA*32 for reduction warp aw of NA) and walk the
-// tensors in processing order, 16 loads in flight per lane, folding max |x| on
-// the integer pipe.  Finishing a tensor a, a reduction warp folds its maximum
-// into amax_bits[a] (atomicMax on the bit pattern of a non-negative float) and
-// counts itself in arrived[a] (acquire-release); the last to arrive writes
-// S[a].  A sweep warp entering tensor t waits until all NA reduction warps
-// have arrived for t.  Reduction warps never wait, and the grid is resident
-// (cooperative launch), so every wait ends; each is bounded anyway by the
-// global timer (1 s; status bit 1, the warp stops).  p.wait_extra raises the
-// arrival target: 0 in every real call, the wait self-test uses it.  Tensors are processed in ascending size, so the first
-// reduction, the only one no sweep hides, is the smallest.
+// In-launch global scales (cooperative launch, two phases).  Phase 1: every
+// warp of the grid folds max |x| over its share of every tensor (16 loads in
+// flight per lane, on the integer pipe: with the sign bit cleared the unsigned
+// order of bf16/fp32 bit patterns is the order of the magnitudes) and
+// publishes it with an atomicMax on the bit pattern.  A grid barrier (an
+// acquire-release arrival count in the caller's workspace, zeroed by a
+// memset before the launch; bounded by the global timer, 1 s, then status bit
+// 1) separates it from phase 2, the sweep, which reads S[t] = fl(amax_t /
+// fl(6 D)).  The reduction is HBM-bound and the sweep FP32-bound; running them
+// one after the other keeps the sweep at 8 warps per CTA and the full
+// register budget.  (A ninth, reduction-only warp per CTA that overlapped
+// tensor t+1's reduction with tensor t's sweep capped every thread at 96
+// registers and interfered with the sweep's loads; on the two 242M-element
+// matrices of the Qwen2.5-72B shapes, where only half the data can overlap
+// at all, it measured 1.674 ms against 1.409 ms for the sweep alone.)
 #include <atomic>
 
 #include "group_kernels.h"
@@ -101,40 +101,20 @@ __device__ __noinline__ float rescan_share(const uint4* xv, int64_t nvec, int64_
     return m;
 }
 
+// Phase 1 of a dynamic-scale launch: every warp of the grid folds max |x| over
+// its share of every tensor (vector w*32 + lane + j*W*32 for warp w of W, 16
+// loads in flight per lane) and publishes it with an atomicMax on the bit
+// pattern; a share holding a NaN is rescanned with the NaN-skipping float
+// max, so S matches the two-launch path bit for bit, and sets status bit 0
+// for NaN/inf.  Each warp's atomics are fenced before the CTA arrives at the
+// grid barrier.
 template <int DT>
-__device__ __forceinline__ void publish_max(const GroupParams& p, int a, uint32_t m, const uint4* xv, int64_t nvec,
-                                            int64_t first, int64_t step, int lane) {
-    uint32_t mbits;
-    bool nan, inf;
-    if (DT == 0) {
-        const uint32_t M = max(m & 0xFFFFu, m >> 16);
-        nan = M > 0x7F80u;
-        inf = M == 0x7F80u;
-        mbits = M << 16;
-    } else {
-        nan = m > 0x7F800000u;
-        inf = m == 0x7F800000u;
-        mbits = m;
-    }
-    if (__any_sync(0xffffffffu, nan)) mbits = __float_as_uint(rescan_share<DT>(xv, nvec, first, step));
-    const unsigned mb = __reduce_max_sync(0xffffffffu, mbits);
-    const bool bad = __any_sync(0xffffffffu, nan || inf);
-    if (lane == 0) {
-        if (mb) atomicMax(p.amax_bits + a, mb);
-        if (bad && p.status_dev) atomicOr(p.status_dev, 1);
-        const unsigned old = atom_add_acq_rel(p.arrived + a, 1u);
-        if (old == gridDim.x - 1) {
-            const float amax = __uint_as_float(ld_relaxed_u32(p.amax_bits + a));
-            p.S[p.t[a].s_index] = __fdiv_rn(amax, __fmul_rn(6.0f, p.fp8_div));
-        }
-    }
-}
-
-// One reduction warp (aw = blockIdx.x of NA = gridDim.x): its share of every
-// tensor, in processing order, vector aw*32 + lane + j*NA*32 for round j.
-template <int DT>
-__device__ __forceinline__ void reduce_warp(const GroupParams& p, int lane) {
-    const int64_t aw = blockIdx.x, step = (int64_t)gridDim.x * 32, first = aw * 32 + lane;
+__device__ __forceinline__ void reduce_all(const GroupParams& p) {
+    const int lane = threadIdx.x & 31;
+    const int64_t W = (int64_t)gridDim.x * (kSweepThreads / 32);
+    const int64_t w = (int64_t)blockIdx.x * (kSweepThreads / 32) + (threadIdx.x >> 5);
+    const int64_t step = W * 32, first = w * 32 + lane;
+    bool any_bad = false;
     for (int a = 0; a < p.count; a++) {
         const uint4* xv = static_cast<const uint4*>(p.t[a].x);
         const int64_t nvec = p.t[a].nvec;
@@ -148,8 +128,53 @@ __device__ __forceinline__ void reduce_warp(const GroupParams& p, int lane) {
             for (int i = 0; i < kAmaxInFlight; i++) m = fold_vec<DT>(m, u[i]);
         }
         for (; v < nvec; v += step) m = fold_vec<DT>(m, ld_stream16(xv + v));
-        publish_max<DT>(p, a, m, xv, nvec, first, step, lane);
+        uint32_t mbits;
+        bool nan, inf;
+        if (DT == 0) {
+            const uint32_t M = max(m & 0xFFFFu, m >> 16);
+            nan = M > 0x7F80u;
+            inf = M == 0x7F80u;
+            mbits = M << 16;
+        } else {
+            nan = m > 0x7F800000u;
+            inf = m == 0x7F800000u;
+            mbits = m;
+        }
+        if (__any_sync(0xffffffffu, nan)) mbits = __float_as_uint(rescan_share<DT>(xv, nvec, first, step));
+        const unsigned mb = __reduce_max_sync(0xffffffffu, mbits);
+        any_bad |= __any_sync(0xffffffffu, nan || inf);
+        if (lane == 0 && mb) atomicMax(p.amax_bits + a, mb);
     }
+    if (lane == 0) {
+        if (any_bad && p.status_dev) atomicOr(p.status_dev, 1);
+        __threadfence();
+    }
+}
+
+// Grid barrier between the two phases (cooperative launch: every CTA is
+// resident, so the count always completes; the wait is bounded anyway by the
+// global timer, 1 s, after which bit 1 of the status word is set and the
+// launch returns without writing outputs).  p.wait_extra raises the target:
+// 0 in every real call, the wait self-test uses it.
+__device__ __forceinline__ bool grid_barrier(const GroupParams& p) {
+    __shared__ int s_timeout;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        atom_add_acq_rel(p.arrived, 1u);
+        const unsigned long long t0 = global_ns();
+        int timeout = 0;
+        while (ld_acquire_u32(p.arrived) < gridDim.x + p.wait_extra) {
+            if (global_ns() - t0 > kGroupWaitNs) {
+                timeout = 1;
+                break;
+            }
+            __nanosleep(128);
+        }
+        s_timeout = timeout;
+        if (timeout && p.status_dev) atomicOr(p.status_dev, 2);
+    }
+    __syncthreads();
+    return !s_timeout;
 }
 
 // One 16-element segment of the grid-stride loop: ScaleSweep (METHOD 0,
@@ -272,25 +297,27 @@ __device__ __forceinline__ int tensor_at(const GroupParams& p, int t, int64_t se
     return t;
 }
 
-// DYN = 0: static scales read from p.S, 8 sweep warps per CTA; DYN = 1:
-// scales reduced in the launch by a ninth warp per CTA.  (Nine warps cap the
-// registers at 96 per thread -- two CTAs put five warps on two schedulers --
-// which measured faster than seven sweep warps plus one reduction warp.)
+// DYN = 0: static scales read from p.S.  DYN = 1: the scales are reduced in
+// the launch first (phase 1, every warp, HBM-bound), then every CTA meets at
+// a grid barrier and sweeps with the same 8 warps (phase 2, FP32-bound).
 template <int DT, int METHOD, int OBJ, int BLOCK, int DYN>
-__global__ void __launch_bounds__(DYN ? kSweepThreads + 32 : kSweepThreads, NVFP4_GROUP_MINB)
+__global__ void __launch_bounds__(kSweepThreads, NVFP4_GROUP_MINB)
     quantize_group_kernel(const __grid_constant__ GroupParams p) {
     constexpr int SW = kSweepThreads;
     static_assert(SW == kGroupCtaSegments, "host padding unit");
     __shared__ Cand tab[kTabN];
     build_table(tab);
-    __syncthreads();
-    if (DYN && threadIdx.x >= SW) {
-        reduce_warp<DT>(p, threadIdx.x & 31);
-        return;
+    if (DYN) {
+        reduce_all<DT>(p);
+        if (!grid_barrier(p)) return;
+        if (blockIdx.x == 0 && (int)threadIdx.x < p.count)        // publish every tensor's S once
+            p.S[p.t[threadIdx.x].s_index] =
+                __fdiv_rn(__uint_as_float(ld_relaxed_u32(p.amax_bits + threadIdx.x)), __fmul_rn(6.0f, p.fp8_div));
     }
+    __syncthreads();
 
     const int count = p.count;
-    const int tid = threadIdx.x, lane = tid & 31;
+    const int tid = threadIdx.x;
     const int64_t stride = (int64_t)gridDim.x * SW;
     const int64_t total = p.total_seg;
     int64_t cbase = (int64_t)blockIdx.x * SW;
@@ -307,29 +334,9 @@ __global__ void __launch_bounds__(DYN ? kSweepThreads + 32 : kSweepThreads, NVFP
     }
 
     while (cbase < total) {
-        // entering tensor t: its global scale (dynamic: once every reduction
-        // warp has arrived for t)
-        float S;
-        if (DYN) {
-            int timeout = 0;
-            if (lane == 0) {
-                const unsigned long long t0 = global_ns();
-                while (ld_acquire_u32(p.arrived + t) < gridDim.x + p.wait_extra) {
-                    if (global_ns() - t0 > kGroupWaitNs) {
-                        timeout = 1;
-                        break;
-                    }
-                    __nanosleep(128);
-                }
-            }
-            if (__shfl_sync(0xffffffffu, timeout, 0)) {
-                if (lane == 0 && p.status_dev) atomicOr(p.status_dev, 2);
-                return;
-            }
-            S = __fdiv_rn(__uint_as_float(ld_relaxed_u32(p.amax_bits + t)), __fmul_rn(6.0f, p.fp8_div));
-        } else {
-            S = __ldg(p.S + p.t[t].s_index);
-        }
+        // entering tensor t: its global scale
+        const float S = DYN ? __fdiv_rn(__uint_as_float(ld_relaxed_u32(p.amax_bits + t)), __fmul_rn(6.0f, p.fp8_div))
+                            : __ldg(p.S + p.t[t].s_index);
         float E = __frcp_rn(S);
         const bool usable = (S > 0.0f) && isfinite(S) && isfinite(E);
         if (!usable) E = 1.0f;
@@ -362,7 +369,7 @@ namespace {
 
 template <int DT, int METHOD, int OBJ, int BLOCK, int DYN>
 cudaError_t launch_group(const GroupParams& p, int sms, cudaStream_t s) {
-    constexpr int SW = kSweepThreads, threads = DYN ? kSweepThreads + 32 : kSweepThreads;
+    constexpr int SW = kSweepThreads, threads = kSweepThreads;
     constexpr int SEGS = BLOCK / 16;
     static std::atomic<int> occ_cache[kOccDevices];
     const int64_t cap = (int64_t)sms *
