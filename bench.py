@@ -637,9 +637,13 @@ def run_kernel_case(args):
         # scales), or a slice of each (2048 and 7392 leading rows: 242 MB of
         # inputs, still above L2) for profiler captures
         from paper_2606_07618_gb300 import step as ST
-        wlq, qx, qw = load_workload(WORKLOAD, dev)
         if args.kernel_case.startswith("qwen_slice"):
-            qx = [qx[0][:2048], qx[1][:7392]]
+            from paper_2606_07618_gb300 import workloads as W
+            wlq = W.workload(WORKLOAD)
+            qx = [W.draw(t, rows=slice(0, r)).to(dev) for t, r in zip(wlq.tensors, (2048, 7392))]
+            qw = [W.draw_weights(t).to(dev) for t in wlq.tensors]
+        else:
+            wlq, qx, qw = load_workload(WORKLOAD, dev)
         sq = ST.for_workload(wlq, qx, qw)
         fns["qwen_group"] = fns["qwen_slice_group"] = lambda: sq()
         fns["qwen_absmax_group"] = fns["qwen_slice_absmax_group"] = lambda: sq.absmax()

@@ -380,6 +380,40 @@ nvfp4_status ldlq_quantize(const void* W, nvfp4_dtype dt, int64_t rows, int64_t 
                            const uint8_t* sf_linear, const int32_t* perm, const float* U, uint8_t* codes,
                            int* status_dev, void* workspace, size_t ws_bytes, void* stream);
 
+/*
+ * Row partition of one [rows, cols] tensor over `world` shards (ranks, GPUs)
+ * for the multi-GPU path: given S every block is independent (Sec. 4.2.1), so
+ * shard `rank` quantises rows [row_begin, row_end) alone, with the global
+ * scale S = fl32(max_k amax_k / fl32(6 D)) taken as the maximum of the shards'
+ * own nvfp4_global_scale results (one max-allreduce of a float: fl32(a/c) is
+ * monotone in a, so the maximum of the shards' S is the whole tensor's S, bit
+ * for bit; OR-reduce the status words too).  Shard boundaries fall on
+ * multiples of 128 rows, so no 128x4 swizzled-scale atom straddles two shards
+ * and each shard's outputs are contiguous byte ranges of the whole tensor's:
+ * calling scalesweep_quantize (or any quantisation call) on the shard's rows
+ * with these offsets added to the whole tensor's output pointers writes
+ * exactly the bytes the single call would.  Row blocks of 128 are split as
+ * evenly as possible; a shard may be empty (row_begin == row_end) when world
+ * exceeds the row blocks.  Host-only: no CUDA call, no device access.
+ *   block        16, 32 or 64; the swizzled offsets are -1 unless block == 16.
+ *   out          receives the shard's rows and offsets (elements for x, bytes
+ *                for the outputs).
+ * Returns NVFP4_ERR_INVALID_ARG for a null `out`, world < 1 or rank outside
+ * [0, world), and the shape errors of scalesweep_quantize.  The paper has no
+ * counterpart: it states the independence the partition relies on.
+ */
+typedef struct {
+    int64_t row_begin, row_end;     /* the shard's rows */
+    int64_t x_offset;               /* elements: row_begin * cols */
+    int64_t codes_offset;           /* bytes: row_begin * cols / 2 */
+    int64_t sf_linear_offset;       /* bytes: row_begin * cols / block */
+    int64_t sf_swizzled_offset;     /* bytes: (row_begin / 128) * ceil(cols/64) * 512, or -1 */
+    int64_t sf_swizzled_bytes;      /* the shard's swizzled extent, or -1 */
+} nvfp4_row_shard;
+
+nvfp4_status nvfp4_row_shard_layout(int64_t rows, int64_t cols, int block, int world, int rank,
+                                    nvfp4_row_shard* out);
+
 #ifdef __cplusplus
 }
 #endif

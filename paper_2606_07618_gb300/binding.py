@@ -36,6 +36,13 @@ _lib = None
 NVFP4_GROUP_MAX = 16
 
 
+class RowShard(ctypes.Structure):
+    """nvfp4_row_shard: one shard's rows and output offsets (nvfp4_row_shard_layout)."""
+    _fields_ = [("row_begin", ctypes.c_int64), ("row_end", ctypes.c_int64), ("x_offset", ctypes.c_int64),
+                ("codes_offset", ctypes.c_int64), ("sf_linear_offset", ctypes.c_int64),
+                ("sf_swizzled_offset", ctypes.c_int64), ("sf_swizzled_bytes", ctypes.c_int64)]
+
+
 class GroupTensor(ctypes.Structure):
     """nvfp4_group_tensor: one tensor of a scalesweep_quantize_group call."""
     _fields_ = [("x", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64), ("w", ctypes.c_void_p),
@@ -72,6 +79,7 @@ def lib() -> ctypes.CDLL:
         L.scalesweep_quantize_group.argtypes = [ctypes.POINTER(GroupTensor), i, i, i, i, f, p, p, p, sz, p]
         L.absmax_quantize_group.argtypes = [ctypes.POINTER(GroupTensor), i, i, i, f, p, p, p, sz, p]
         L.nvfp4_selftest_wait_timeout.argtypes = [i, p, i64, i64, p, p, p, sz, p, p, p]
+        L.nvfp4_row_shard_layout.argtypes = [i64, i64, i, i, i, ctypes.POINTER(RowShard)]
         L.nvfp4_optimal_scale.argtypes = [p, i, i64, i64, i, p, i, p, i64, p, p, p, p, p]
         L.nvfp4_ldlq_prepare_workspace.argtypes, L.nvfp4_ldlq_prepare_workspace.restype = [i64], sz
         L.nvfp4_ldlq_prepare.argtypes = [p, i64, f, p, p, p, p, p, sz, p]
@@ -80,7 +88,8 @@ def lib() -> ctypes.CDLL:
         for fn in ("nvfp4_global_scale", "nvfp4_global_scale_noalloc", "scalesweep_quantize", "absmax_quantize",
                    "four_over_six_quantize", "nvfp4_dequantize", "scalesweep_quantize_dynamic",
                    "absmax_quantize_dynamic", "nvfp4_optimal_scale", "nvfp4_ldlq_prepare", "ldlq_quantize",
-                   "scalesweep_quantize_group", "absmax_quantize_group", "nvfp4_selftest_wait_timeout"):
+                   "scalesweep_quantize_group", "absmax_quantize_group", "nvfp4_selftest_wait_timeout",
+                   "nvfp4_row_shard_layout"):
             getattr(L, fn).restype = i
         _lib = L
     return _lib
@@ -295,3 +304,11 @@ def ldlq_quantize(W, block: int, S, sf_linear, perm, U, codes, status=None, work
     rc = lib().ldlq_quantize(_ptr(W), _dtype(W), rows, cols, int(block), _ptr(S), _ptr(sf_linear), _ptr(perm),
                              _ptr(U), _ptr(codes), _ptr(status), _ptr(workspace), ws_bytes, _stream(stream))
     _check("ldlq_quantize", rc)
+
+
+def nvfp4_row_shard_layout(rows: int, cols: int, block: int, world: int, rank: int) -> RowShard:
+    """Rows and output offsets of shard `rank` of `world` (host-only, no GPU needed)."""
+    out = RowShard()
+    rc = lib().nvfp4_row_shard_layout(int(rows), int(cols), int(block), int(world), int(rank), ctypes.byref(out))
+    _check("nvfp4_row_shard_layout", rc)
+    return out

@@ -620,4 +620,29 @@ nvfp4_status ldlq_quantize(const void* W, nvfp4_dtype dt, int64_t rows, int64_t 
     return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
 }
 
+nvfp4_status nvfp4_row_shard_layout(int64_t rows, int64_t cols, int block, int world, int rank,
+                                    nvfp4_row_shard* out) {
+    if (!out || world < 1 || rank < 0 || rank >= world) return NVFP4_ERR_INVALID_ARG;
+    Shape sh;
+    const nvfp4_status st = check_shape(rows, cols, block, &sh);
+    if (st != NVFP4_OK) return st;
+    const int64_t rb = (rows + 127) / 128;                       // row blocks of 128
+    if (rb > INT64_MAX / world) return NVFP4_ERR_RANGE;
+    const int64_t b0 = rb * rank / world, b1 = rb * (rank + 1) / world;
+    const int64_t r0 = b0 * 128 < rows ? b0 * 128 : rows, r1 = b1 * 128 < rows ? b1 * 128 : rows;
+    out->row_begin = r0;
+    out->row_end = r1;
+    out->x_offset = r0 * cols;
+    out->codes_offset = r0 * cols / 2;
+    out->sf_linear_offset = r0 * sh.kb;
+    if (block == 16) {
+        out->sf_swizzled_offset = b0 * sh.kpad4 * 512;
+        out->sf_swizzled_bytes = (b1 - b0) * sh.kpad4 * 512;
+    } else {
+        out->sf_swizzled_offset = -1;
+        out->sf_swizzled_bytes = -1;
+    }
+    return NVFP4_OK;
+}
+
 }  // extern "C"

@@ -108,7 +108,7 @@ __device__ __noinline__ float rescan_share(const uint4* xv, int64_t nvec, int64_
 // max, so S matches the two-launch path bit for bit, and sets status bit 0
 // for NaN/inf.  Each warp's atomics are fenced before the CTA arrives at the
 // grid barrier.
-template <int DT>
+template <int DT, int INFLIGHT>
 __device__ __forceinline__ void reduce_all(const GroupParams& p) {
     const int lane = threadIdx.x & 31;
     const int64_t W = (int64_t)gridDim.x * (kSweepThreads / 32);
@@ -120,12 +120,12 @@ __device__ __forceinline__ void reduce_all(const GroupParams& p) {
         const int64_t nvec = p.t[a].nvec;
         uint32_t m = 0;
         int64_t v = first;
-        for (; v + (kAmaxInFlight - 1) * step < nvec; v += kAmaxInFlight * step) {
-            uint4 u[kAmaxInFlight];
+        for (; v + (INFLIGHT - 1) * step < nvec; v += INFLIGHT * step) {
+            uint4 u[INFLIGHT];
 #pragma unroll
-            for (int i = 0; i < kAmaxInFlight; i++) u[i] = ld_stream16(xv + v + i * step);
+            for (int i = 0; i < INFLIGHT; i++) u[i] = ld_stream16(xv + v + i * step);
 #pragma unroll
-            for (int i = 0; i < kAmaxInFlight; i++) m = fold_vec<DT>(m, u[i]);
+            for (int i = 0; i < INFLIGHT; i++) m = fold_vec<DT>(m, u[i]);
         }
         for (; v < nvec; v += step) m = fold_vec<DT>(m, ld_stream16(xv + v));
         uint32_t mbits;
@@ -300,15 +300,22 @@ __device__ __forceinline__ int tensor_at(const GroupParams& p, int t, int64_t se
 // DYN = 0: static scales read from p.S.  DYN = 1: the scales are reduced in
 // the launch first (phase 1, every warp, HBM-bound), then every CTA meets at
 // a grid barrier and sweeps with the same 8 warps (phase 2, FP32-bound).
+// AbsMax is HBM-bound in both phases: it is held to 64 registers (4 CTAs per
+// SM, 8 loads in flight per lane in phase 1) for more loads in flight.
+template <int METHOD>
+constexpr int group_min_blocks() {
+    return METHOD == 1 ? 4 : NVFP4_GROUP_MINB;
+}
+
 template <int DT, int METHOD, int OBJ, int BLOCK, int DYN>
-__global__ void __launch_bounds__(kSweepThreads, NVFP4_GROUP_MINB)
+__global__ void __launch_bounds__(kSweepThreads, group_min_blocks<METHOD>())
     quantize_group_kernel(const __grid_constant__ GroupParams p) {
     constexpr int SW = kSweepThreads;
     static_assert(SW == kGroupCtaSegments, "host padding unit");
     __shared__ Cand tab[kTabN];
     build_table(tab);
     if (DYN) {
-        reduce_all<DT>(p);
+        reduce_all<DT, METHOD == 1 ? 8 : kAmaxInFlight>(p);
         if (!grid_barrier(p)) return;
         if (blockIdx.x == 0 && (int)threadIdx.x < p.count)        // publish every tensor's S once
             p.S[p.t[threadIdx.x].s_index] =

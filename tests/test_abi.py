@@ -31,7 +31,7 @@ def test_header_declares_the_api():
         "nvfp4_dynamic_workspace", "scalesweep_quantize_dynamic", "absmax_quantize_dynamic",
         "nvfp4_optimal_scale", "nvfp4_ldlq_prepare_workspace", "nvfp4_ldlq_prepare", "nvfp4_ldlq_workspace",
         "ldlq_quantize", "scalesweep_quantize_group_workspace", "scalesweep_quantize_group",
-        "absmax_quantize_group", "nvfp4_selftest_wait_timeout"])
+        "absmax_quantize_group", "nvfp4_selftest_wait_timeout", "nvfp4_row_shard_layout"])
 
 
 def test_library_exports_every_declared_symbol(L):
@@ -182,8 +182,9 @@ def test_group_validation_without_gpu(L):
 
 def test_header_constants_and_struct_layout_match_the_binding(tmp_path):
     """Compile a C probe against include/nvfp4ss.h with the host C compiler and
-    compare the enum values, the window and group constants and the layout of
-    nvfp4_group_tensor with what the Python binding passes through ctypes."""
+    compare the enum values, the window and group constants and the layouts of
+    nvfp4_group_tensor and nvfp4_row_shard with what the Python binding passes
+    through ctypes."""
     import shutil
     import subprocess
     from paper_2606_07618_gb300 import binding as B
@@ -195,9 +196,13 @@ def test_header_constants_and_struct_layout_match_the_binding(tmp_path):
 #include <stdio.h>
 #include "nvfp4ss.h"
 #define F(name) printf(#name " %zu %zu\n", offsetof(nvfp4_group_tensor, name), sizeof(((nvfp4_group_tensor*)0)->name))
+#define R(name) printf("shard_" #name " %zu %zu\n", offsetof(nvfp4_row_shard, name), sizeof(((nvfp4_row_shard*)0)->name))
 int main(void) {
     printf("size %zu\n", sizeof(nvfp4_group_tensor));
     F(x); F(rows); F(cols); F(w); F(w_row_stride); F(codes); F(sf_linear); F(sf_swizzled);
+    printf("shard_size %zu\n", sizeof(nvfp4_row_shard));
+    R(row_begin); R(row_end); R(x_offset); R(codes_offset); R(sf_linear_offset); R(sf_swizzled_offset);
+    R(sf_swizzled_bytes);
     printf("NVFP4_IN_BF16 %d\nNVFP4_IN_F32 %d\nNVFP4_OBJ_MSE %d\nNVFP4_OBJ_WMSE %d\n", NVFP4_IN_BF16, NVFP4_IN_F32,
            NVFP4_OBJ_MSE, NVFP4_OBJ_WMSE);
     printf("NVFP4_SF_LINEAR %d\nNVFP4_SF_SWIZZLED %d\n", NVFP4_SF_LINEAR, NVFP4_SF_SWIZZLED);
@@ -214,6 +219,10 @@ int main(void) {
     for name, _ in B.GroupTensor._fields_:
         f = getattr(B.GroupTensor, name)
         assert vals[name] == [f.offset, f.size], name
+    assert vals["shard_size"] == [ctypes.sizeof(B.RowShard)]
+    for name, _ in B.RowShard._fields_:
+        f = getattr(B.RowShard, name)
+        assert vals["shard_" + name] == [f.offset, f.size], name
     for name in ("NVFP4_IN_BF16", "NVFP4_IN_F32", "NVFP4_OBJ_MSE", "NVFP4_OBJ_WMSE", "NVFP4_SF_LINEAR",
                  "NVFP4_SF_SWIZZLED", "NVFP4_WINDOW_DEFAULT", "NVFP4_WINDOW_TIGHT", "NVFP4_GROUP_MAX"):
         assert vals[name] == [getattr(B, name)], name
@@ -234,7 +243,11 @@ def _ctype_of(param):
     from paper_2606_07618_gb300 import binding as B
     decl = param.rsplit(None, 1)[0] if not param.endswith("*") else param
     if "*" in param:
-        return ctypes.POINTER(B.GroupTensor) if "nvfp4_group_tensor" in param else ctypes.c_void_p
+        if "nvfp4_group_tensor" in param:
+            return ctypes.POINTER(B.GroupTensor)
+        if "nvfp4_row_shard" in param:
+            return ctypes.POINTER(B.RowShard)
+        return ctypes.c_void_p
     t = decl.replace("const", "").strip()
     return {"int": ctypes.c_int, "int64_t": ctypes.c_int64, "float": ctypes.c_float, "size_t": ctypes.c_size_t,
             "nvfp4_dtype": ctypes.c_int, "nvfp4_objective": ctypes.c_int, "nvfp4_sf_layout": ctypes.c_int,
