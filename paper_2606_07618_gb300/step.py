@@ -1,13 +1,13 @@
 """One pass of the hot path over a set of tensors, through the C ABI.
 
-``QuantizeStep`` owns the output buffers for a list of device tensors and
+``QuantizeStep`` owns the output buffers for a list of tensors and
 quantises all of them with ONE library call per step: the per-call global
 scale of every tensor (S = amax / (6 D), Sec. 4.2.1) and the ScaleSweep of
 every block (Sec. 4.2.2), writing packed E2M1 codes and E4M3 scales.
 
   * several tensors, or a single weight: ``scalesweep_quantize_group`` with
     in-launch scales (a layer's weights, the KV-cache/query tensors, ...);
-  * a single activation tensor (``dynamic=True``): the fused
+  * a single activation tensor (``activation=True``): the fused
     ``scalesweep_quantize_dynamic`` (amax and sweep in one cooperative launch).
 
 ``absmax`` runs the AbsMax baseline (Sec. 3.2) over the same tensors in the
@@ -24,7 +24,13 @@ from . import binding as B
 
 class QuantizeStep:
     def __init__(self, xs, ws=None, block: int = 16, objective: int = B.NVFP4_OBJ_MSE, fp8_div: float = 256.0,
-                 activation: bool = False, swizzled: bool | None = None, w_row_strides=None):
+                 activation: bool = False, swizzled: bool | None = None, w_row_strides=None, outs=None,
+                 device=None):
+        """xs: tensors the GPU can read (device memory, or pinned host memory
+        the kernels then read over the host link); outs: optional output dicts
+        as from binding.empty_outputs (e.g. pinned host memory), else device
+        buffers are allocated; device: where S, the status word and the
+        workspace live (default: the device of xs[0])."""
         if not xs:
             raise ValueError("QuantizeStep needs at least one tensor")
         self.xs = list(xs)
@@ -33,11 +39,12 @@ class QuantizeStep:
         self.objective = int(objective)
         self.fp8_div = float(fp8_div)
         self.fused = bool(activation) and len(self.xs) == 1
-        dev = self.xs[0].device
+        dev = torch.device(device) if device is not None else self.xs[0].device
         if swizzled is None:
             swizzled = self.block == 16
-        self.outs = [B.empty_outputs(x.shape[0], x.shape[1], self.block, device=dev, linear=True, swizzled=swizzled)
-                     for x in self.xs]
+        self.outs = list(outs) if outs is not None else [
+            B.empty_outputs(x.shape[0], x.shape[1], self.block, device=dev, linear=True, swizzled=swizzled)
+            for x in self.xs]
         self.S = torch.empty(len(self.xs), dtype=torch.float32, device=dev)
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         self.dtype = B.NVFP4_IN_BF16 if self.xs[0].dtype == torch.bfloat16 else B.NVFP4_IN_F32

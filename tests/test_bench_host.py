@@ -89,7 +89,7 @@ def test_traffic_record_is_dropped_when_sources_change(tmp_path, monkeypatch):
 
 
 def test_committed_traffic_records_are_well_formed():
-    for name in ("quantize_group_kernel_wmse_traffic.json", "quantize_kernel_wmse_traffic.json"):
+    for name in ("quantize_group_kernel_qwen72b_traffic.json",):
         with open(os.path.join(bench.ROOT, "profiles", name)) as f:
             rec = json.load(f)
         assert rec["source_files"] and len(rec["source_sha256"]) == 64
@@ -98,6 +98,34 @@ def test_committed_traffic_records_are_well_formed():
         assert 1.0 < rec["dram_bytes_per_element"] < 6.0
         for fn in rec["source_files"]:
             assert os.path.exists(os.path.join(bench.ROOT, fn)), fn
+
+
+def test_workload_roofline_terms():
+    """Candidates per block, FP32 ops per element and algorithmic HBM bytes of a
+    step with in-launch scales (two input reads, codes, scales, weights)."""
+    from paper_2606_07618_gb300 import workloads as W
+
+    class T:                                 # stand-in for a device tensor: shape, numel, element size
+        def __init__(self, r, c):
+            self.shape = (r, c)
+
+        def numel(self):
+            return self.shape[0] * self.shape[1]
+
+        def element_size(self):
+            return 2
+    wl = W.workload("qwen72b-b16-wmse")
+    xs = [T(t.rows, t.cols) for t in wl.tensors]
+    assert bench.candidates(wl) == 16 and bench.alu_ops_per_elem(wl) == 64
+    n = 2 * 8192 * 29568
+    assert bench.hbm_bytes(wl, xs) == n * (2 + 2 + 0.5 + 2 / 16) + 4 * (29568 + 8192)
+    wl = W.workload("qwen72b-b16-mse")
+    assert bench.candidates(wl) == 11 and bench.alu_ops_per_elem(wl) == 33
+    wl = W.workload("qwen72b-b64-mse")
+    assert bench.candidates(wl) == 16 and bench.alu_ops_per_elem(wl) == 48
+    assert bench.hbm_bytes(wl, xs) == n * (2 + 2 + 0.5 + 1 / 64)
+    assert bench.WORKLOAD == "qwen72b-b16-wmse"
+    assert sorted(bench.LEG_CONFIGS + [bench.WORKLOAD]) == sorted(W.ALL_CONFIGS)
 
 
 def test_algorithmic_bytes_per_element():

@@ -329,3 +329,30 @@ def test_group_dynamic_in_cuda_graph(B):
         for a, b in zip(outs, outs2):
             for k in ("codes", "sf_linear", "sf_swizzled"):
                 assert torch.equal(a[k], b[k])
+
+
+@pytest.mark.parametrize("activation", [False, True])
+def test_zero_copy_host_buffers_equal_device_buffers(B, activation):
+    """Inputs and outputs in pinned host memory (the kernels load and store over
+    the host link): the same bytes as with device buffers, for the grouped
+    launch and for the fused single-tensor launch."""
+    from paper_2606_07618_gb300 import step as ST
+    shapes = [(300, 512)] if activation else [(300, 512), (130, 192), (64, 1024)]
+    xs = [W.small_tensor(r, c, 40 + i, dist="student_t", std=1.0, outliers=2, mult=30.0) for i, (r, c) in
+          enumerate(shapes)]
+    ws = [torch.exp(torch.randn(c, generator=torch.Generator().manual_seed(i))).to(DEV) for i, (_, c) in
+          enumerate(shapes)]
+    obj = B.NVFP4_OBJ_WMSE
+    dev_step = ST.QuantizeStep([x.to(DEV) for x in xs], ws, objective=obj, activation=activation)
+    hx = [x.pin_memory() for x in xs]
+    houts = [{k: torch.empty_like(v, device="cpu").pin_memory() if v is not None else None for k, v in o.items()}
+             for o in dev_step.outs]
+    host_step = ST.QuantizeStep(hx, ws, objective=obj, activation=activation, outs=houts, device=DEV)
+    dev_step()
+    host_step()
+    torch.cuda.synchronize()
+    assert torch.equal(dev_step.S, host_step.S) and host_step.status.item() == 0
+    for a, b in zip(dev_step.outs, houts):
+        for k in ("codes", "sf_linear", "sf_swizzled"):
+            assert torch.equal(a[k].cpu(), b[k]), k
+
