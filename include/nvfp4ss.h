@@ -346,8 +346,13 @@ nvfp4_status nvfp4_dequantize(const uint8_t* codes, const uint8_t* sf, nvfp4_sf_
  *           positive definite or has a non-finite diagonal (a failing pivot is
  *           replaced by 1 so the outputs stay finite, but they are not a
  *           factorization then).
+ *           |= 16 if a tensor-core update's bounded wait ran out (about a
+ *           second; that update is then not applied).
  *   workspace   device bytes, at least nvfp4_ldlq_prepare_workspace(n).
- * Cost: n^3/3 fp32 multiply-adds (blocked Cholesky, 64-wide panels).
+ * Cost: n^3/3 fp32 multiply-adds (blocked Cholesky, 64-wide panels).  The
+ * trailing updates run on the tensor cores as three TF32 products per term
+ * (products to ~2^-21 relative, accumulated in fp32) when n % 4 == 0 and H,
+ * U are 16-byte aligned, else on the FP32 pipe.
  * The factorization's critical chain runs on a high-priority stream the library
  * creates on the first call on a device and keeps (with four events) for the
  * process; it is forked from and joined back into `stream`, so the call stays
@@ -367,6 +372,10 @@ nvfp4_status nvfp4_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* 
  * U_ik, What_k = Q(T_k), with Q the sweep's fp32 rounding at the fixed scale:
  * y = fl(T*E), q = RNE_E2M1(fl(y*fl(1/v))), What = fl(fl(q*v)*S); a zero scale
  * code or an unusable S quantizes to signed zeros, an exactly zero y to +0.
+ *   The error-feedback updates run on the tensor cores (three TF32 products
+ *   per term, as in nvfp4_ldlq_prepare; status bit 16 as there) when rows and
+ *   cols are multiples of 4 and the buffers 16-byte aligned, else on the FP32
+ *   pipe.
  *   perm, U from nvfp4_ldlq_prepare (cols = n); status_dev optional: |= 8 if
  *   perm holds an index outside [0, cols) (the entry is then read as 0).
  *   workspace   device bytes, at least nvfp4_ldlq_workspace(rows, cols):

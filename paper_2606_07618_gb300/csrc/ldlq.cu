@@ -28,6 +28,7 @@
 #include "nvfp4_device.cuh"
 #include "ldlq_kernels.h"
 #include "nvfp4_kernels.h"
+#include "tc_gemm.cuh"
 
 namespace nvfp4 {
 
@@ -374,6 +375,18 @@ cudaError_t launch_gemm(float* C, int64_t ldc, const float* A, int64_t lda, cons
                : launch_gemm_t<AT, BT, LOWER, false>(C, ldc, A, lda, B, ldb, M, N, K, alpha, s);
 }
 
+// C += alpha op(A) op(B) for the LDLQ updates: on the tensor cores (tcgen05,
+// 3xTF32, tc_gemm.cuh) wherever its TMA alignment rules hold (16-byte aligned
+// bases and row strides), else with the SIMT fp32 GEMM above.  AT: A stored
+// [K][M]; BT: B stored [N][K] (the tensor-core GEMM's B_MN is !BT).
+template <bool AT, bool BT, bool LOWER>
+cudaError_t update_gemm(float* C, int64_t ldc, const float* A, int64_t lda, const float* B, int64_t ldb, int64_t M,
+                        int64_t N, int K, float alpha, int* status, cudaStream_t s) {
+    const cudaError_t e = tc::launch_gemm<AT, !BT, LOWER>(C, ldc, A, lda, B, ldb, M, N, K, alpha, status, s);
+    if (e != cudaErrorNotSupported) return e;
+    return launch_gemm<AT, BT, LOWER>(C, ldc, A, lda, B, ldb, M, N, K, alpha, s);
+}
+
 __global__ void diag_d_kernel(const float* A, int64_t n, float* D) {
     const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (k < n) {
@@ -656,12 +669,12 @@ cudaError_t launch_ldlq_prepare(const float* H, int64_t n, float damp, int32_t* 
             if ((e = cudaEventRecord(la->panel_done, c)) != cudaSuccess) return e;
             // the next block column also took the previous panel's rest update
             if (have_rest && (e = cudaStreamWaitEvent(c, la->rest_done, 0)) != cudaSuccess) return e;
-            e = launch_gemm<false, true, true>(C, n, P, n, P, n, rest, nb2, nb, -1.0f, c);
+            e = update_gemm<false, true, true>(C, n, P, n, P, n, rest, nb2, nb, -1.0f, status, c);
             if (e != cudaSuccess) return e;
             if (rest > nb2) {
                 if ((e = cudaStreamWaitEvent(s, la->panel_done, 0)) != cudaSuccess) return e;
-                e = launch_gemm<false, true, true>(C + nb2 * n + nb2, n, P + nb2 * n, n, P + nb2 * n, n, rest - nb2,
-                                                   rest - nb2, nb, -1.0f, s);
+                e = update_gemm<false, true, true>(C + nb2 * n + nb2, n, P + nb2 * n, n, P + nb2 * n, n, rest - nb2,
+                                                   rest - nb2, nb, -1.0f, status, s);
                 if (e != cudaSuccess) return e;
                 if ((e = cudaEventRecord(la->rest_done, s)) != cudaSuccess) return e;
                 have_rest = true;
@@ -751,8 +764,8 @@ cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* 
             if (e != cudaSuccess) return e;
             const int64_t rest_in = s0 + span - (k0 + P);
             if (rest_in > 0) {
-                e = launch_gemm<true, false, false>(p.T + k0 + P, p.n, Ek, p.rows, p.U + k0 * p.n + k0 + P, p.n,
-                                                    p.rows, rest_in, P, 1.0f, c);
+                e = update_gemm<true, false, false>(p.T + k0 + P, p.n, Ek, p.rows, p.U + k0 * p.n + k0 + P, p.n,
+                                                    p.rows, rest_in, P, 1.0f, p.status, c);
                 if (e != cudaSuccess) return e;
             }
         }
@@ -763,14 +776,14 @@ cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* 
             // the next super-panel's columns also took the previous rest update, and
             // that update read the EpT buffer the next super-panel overwrites
             if (have_rest && (e = cudaStreamWaitEvent(c, la->rest_done, 0)) != cudaSuccess) return e;
-            e = launch_gemm<true, false, false>(p.T + s0 + span, p.n, EpT, p.rows, p.U + s0 * p.n + s0 + span, p.n,
-                                                p.rows, next, (int)span, 1.0f, c);
+            e = update_gemm<true, false, false>(p.T + s0 + span, p.n, EpT, p.rows, p.U + s0 * p.n + s0 + span, p.n,
+                                                p.rows, next, (int)span, 1.0f, p.status, c);
             if (e != cudaSuccess) return e;
             if (rest > next) {
                 if ((e = cudaStreamWaitEvent(s, la->panel_done, 0)) != cudaSuccess) return e;
-                e = launch_gemm<true, false, false>(p.T + s0 + span + next, p.n, EpT, p.rows,
+                e = update_gemm<true, false, false>(p.T + s0 + span + next, p.n, EpT, p.rows,
                                                     p.U + s0 * p.n + s0 + span + next, p.n, p.rows, rest - next,
-                                                    (int)span, 1.0f, s);
+                                                    (int)span, 1.0f, p.status, s);
                 if (e != cudaSuccess) return e;
                 if ((e = cudaEventRecord(la->rest_done, s)) != cudaSuccess) return e;
                 have_rest = true;
