@@ -345,6 +345,12 @@ def run_gpu(args, rank, world):
                       "fp32_tops": tp, "fp32_frac": af, "absmax_ms": round(t_ab, 4),
                       "overhead_vs_absmax": round(t_ss / t_ab, 3), "l2": "flushed before each call" if small
                       else "inputs > L2"}
+        if small:                               # the same calls back to back, inputs left in L2
+            t_hot = time_calls(lambda: sc(stream=stream), reps, stream)
+            t_hot_ab = time_calls(lambda: sc.absmax(stream=stream), reps, stream)
+            legs[name]["hot_l2"] = {"ms": round(t_hot, 4), "gelem_s": round(n / (t_hot * 1e-3) / 1e9, 2),
+                                    "absmax_ms": round(t_hot_ab, 4),
+                                    "overhead_vs_absmax": round(t_hot / t_hot_ab, 3)}
         del sc
     _inputs_cache.clear()                       # the headline's tensors stay referenced by xs / ws
 
@@ -534,7 +540,7 @@ def cpu_baseline(wl, xs_cpu, ws_cpu, S_cpu, budget_s=12.0, probe_rows=64):
     threads = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
     obj = oracle.WMSE if wl.objective == "wmse" else oracle.MSE
 
-    def run(rows):
+    def run(rows, nthreads=threads):
         t = time.perf_counter()
         n = 0
         for i, x in enumerate(xs_cpu):
@@ -542,7 +548,7 @@ def cpu_baseline(wl, xs_cpu, ws_cpu, S_cpu, budget_s=12.0, probe_rows=64):
             xs = x[:r].float().numpy()
             S = float(S_cpu[i]) if S_cpu is not None else oracle.global_scale(xs, wl.fp8_div)[0]
             oracle.quantize(0, xs, wl.block, S, obj, w=ws_cpu[i].numpy() if obj == oracle.WMSE else None,
-                            w_row_stride=0, nthreads=threads)
+                            w_row_stride=0, nthreads=nthreads)
             n += xs.size
         return n, time.perf_counter() - t
 
@@ -551,9 +557,14 @@ def cpu_baseline(wl, xs_cpu, ws_cpu, S_cpu, budget_s=12.0, probe_rows=64):
     per_row = sum(x.shape[1] for x in xs_cpu)
     rows = int(max(probe_rows, min(max(x.shape[0] for x in xs_cpu), budget_s * rate / per_row)))
     n, dt = run(rows)
+    # the same oracle on one thread, on a sample of about a tenth of the time
+    rows1 = int(max(8, min(rows, 0.1 * budget_s * (n / dt) / threads / per_row)))
+    n1, dt1 = run(rows1, nthreads=1)
     return {"value": round(n / dt / 1e9, 6), "unit": "Gelem/s", "cores": threads, "kind": "oracle",
             "sample": f"first {rows} rows of each of the {len(xs_cpu)} {wl.name} tensors ({n} elements, "
-                      f"{dt:.1f} s), same S, {wl.objective.upper()}, block {wl.block}"}
+                      f"{dt:.1f} s), same S, {wl.objective.upper()}, block {wl.block}",
+            "one_thread": {"value": round(n1 / dt1 / 1e9, 6), "unit": "Gelem/s", "cores": 1,
+                           "sample": f"first {rows1} rows of each tensor ({n1} elements, {dt1:.1f} s)"}}
 
 
 # ----------------------------------------------------------------------------- reference arm
