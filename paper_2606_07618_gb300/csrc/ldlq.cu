@@ -115,7 +115,8 @@ __global__ void __launch_bounds__(256) gather_h_kernel(const float* H, int64_t n
 // of the 256 threads keeps a 4 x 4 tile in registers.  The pivots stay
 // unscaled, A = M diag(p) M^T with M unit lower triangular: at column j the
 // threads holding column j publish it to shared memory (double-buffered, one
-// barrier per column) and every tile subtracts a_ij a_lj / p_j.  Then
+// barrier per column) and every tile subtracts a_ij a_lj / p_j (rows i > j,
+// columns l > j; the upper parts of the tiles take the same updates unread).  Then
 // L = M diag(sqrt p) and L^-1 = diag(1/sqrt p) M^-1, with M^-1 by forward
 // elimination in the same scheme (column k of M and row k of M^-1 published per
 // step).  A pivot that is not positive and finite sets bit 4 of the status word
@@ -143,47 +144,48 @@ __global__ void __launch_bounds__(256) potrf_kernel(float* A, int64_t n, int64_t
     // row operation X_i -= m_ij X_j (row j of X is final at step j) share one
     // barrier.  Per entry the inverse sees its updates in the order k = 0, 1, ...
     int bad = 0;
-    for (int j = 0; j < kP; j++) {
-        const int b = j & 1;
-        if (c0 <= j && j < c0 + 4) {
+    // columns in groups of four, so that a tile's column j - c0 (and row j - r0)
+    // is a compile-time index: the owners publish without selects
+    for (int jb = 0; jb < kP; jb += 4) {
 #pragma unroll
-            for (int di = 0; di < 4; di++) {
-                const int q = j - c0;
-                const float v = q == 0 ? t[di][0] : q == 1 ? t[di][1] : q == 2 ? t[di][2] : t[di][3];
-                colv[b][r0 + di] = v;
+        for (int q = 0; q < 4; q++) {
+            const int j = jb + q, b = q & 1;
+            if (c0 == jb)
+#pragma unroll
+                for (int di = 0; di < 4; di++) colv[b][r0 + di] = t[di][q];
+            if (r0 == jb)                            // row j of X
+#pragma unroll
+                for (int dc = 0; dc < 4; dc++) rowv[b][c0 + dc] = x[q][dc];
+            __syncthreads();
+            float p = colv[b][j];
+            if (!(p > 0.0f) || !isfinite(p)) {
+                bad = 1;
+                p = 1.0f;
             }
-        }
-        if (r0 <= j && j < r0 + 4) {                 // row j of X
+            if (threadIdx.x == 0) piv[j] = p;
+            const float ip = __frcp_rn(p);
+            const float4 ci = *reinterpret_cast<const float4*>(&colv[b][r0]);
+            const float4 cl = *reinterpret_cast<const float4*>(&colv[b][c0]);
+            const float4 xj = *reinterpret_cast<const float4*>(&rowv[b][c0]);
+            const float civ[4] = {ci.x, ci.y, ci.z, ci.w}, clv[4] = {cl.x, cl.y, cl.z, cl.w};
+            const float xjv[4] = {xj.x, xj.y, xj.z, xj.w};
+            // rows i <= j and columns l <= j take a zero multiplier instead of a
+            // predicate: the skipped terms are exact zeros (the tiles' upper parts
+            // are never read back and stay finite; row j of M^-1 is zero beyond
+            // column j), so all 32 updates run unconditionally
+            float am[4], cm[4];
 #pragma unroll
-            for (int dc = 0; dc < 4; dc++) {
-                const int q = j - r0;
-                const float v = q == 0 ? x[0][dc] : q == 1 ? x[1][dc] : q == 2 ? x[2][dc] : x[3][dc];
-                rowv[b][c0 + dc] = v;
+            for (int d = 0; d < 4; d++) {
+                am[d] = r0 + d > j ? __fmul_rn(civ[d], ip) : 0.0f;
+                cm[d] = c0 + d > j ? clv[d] : 0.0f;
             }
-        }
-        __syncthreads();
-        float p = colv[b][j];
-        if (!(p > 0.0f) || !isfinite(p)) {
-            bad = 1;
-            p = 1.0f;
-        }
-        if (threadIdx.x == 0) piv[j] = p;
-        const float ip = __frcp_rn(p);
-        const float4 ci = *reinterpret_cast<const float4*>(&colv[b][r0]);
-        const float4 cl = *reinterpret_cast<const float4*>(&colv[b][c0]);
-        const float4 xj = *reinterpret_cast<const float4*>(&rowv[b][c0]);
-        const float civ[4] = {ci.x, ci.y, ci.z, ci.w}, clv[4] = {cl.x, cl.y, cl.z, cl.w};
-        const float xjv[4] = {xj.x, xj.y, xj.z, xj.w};
 #pragma unroll
-        for (int di = 0; di < 4; di++) {
-            const int i = r0 + di;
-            const float aij = __fmul_rn(civ[di], ip);
+            for (int di = 0; di < 4; di++)
 #pragma unroll
-            for (int dl = 0; dl < 4; dl++) {
-                const int l = c0 + dl;
-                if (i > j && l > j && l <= i) t[di][dl] = __fmaf_rn(-aij, clv[dl], t[di][dl]);
-                if (i > j && l <= j) x[di][dl] = __fmaf_rn(-aij, xjv[dl], x[di][dl]);
-            }
+                for (int dl = 0; dl < 4; dl++) {
+                    t[di][dl] = __fmaf_rn(-am[di], cm[dl], t[di][dl]);
+                    x[di][dl] = __fmaf_rn(-am[di], xjv[dl], x[di][dl]);
+                }
         }
     }
     __syncthreads();
