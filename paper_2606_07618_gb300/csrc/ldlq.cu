@@ -450,46 +450,58 @@ __global__ void __launch_bounds__(256) gather_w_kernel(LdlqParams p) {
         }
 }
 
-// One LDLQ panel of P <= 64 columns (P % 16 == 0).  Four threads per row
-// (adjacent lanes), thread k of a row owning columns 16k..16k+15 in registers:
-// at column s the owner quantizes it at its fixed scale, writes the error to
-// EpT[s][r], and the error reaches the other three threads by shuffle; each
-// thread then updates its 16 targets through up[s][c] = U[k0+s][k0+c] (zero for
-// c <= s and past the panel).  Splitting the 64-wide update shortens the
-// sequential chain per column four-fold.  The CTA's 32 rows of original weights
-// and scale codes are staged in shared memory with coalesced loads first.
-#ifndef NVFP4_PANEL_TPR
-#define NVFP4_PANEL_TPR 8
-#endif
+// One LDLQ panel of P <= 64 columns (P % 16 == 0).  TPR threads per row
+// (adjacent lanes), thread k of a row owning columns (64/TPR)k .. (64/TPR)(k+1)-1
+// in registers: at column s the owner quantizes it at its fixed scale, writes
+// the error to EpT[s][r], and the error reaches the row's other threads by
+// shuffle; each thread then updates its targets through up[s][c] = U[k0+s][k0+c]
+// (zero for c <= s and past the panel).  Splitting the 64-wide update shortens
+// the sequential chain per column.  The CTA's rows of original weights and the
+// reciprocal and value of each element's scale code are staged in shared memory
+// first, so the owner's step depends on its target alone.  The walk is
+// latency-bound (one dependent quantize -> shuffle -> update chain per column), so
+// weights with few rows take 16 threads per row (twice the warps in flight) and
+// tall ones 8 (fewer shuffles and owner steps per warp).
 constexpr int kPanelThreads = 128;
-constexpr int kPanelTpr = NVFP4_PANEL_TPR;          // threads per row
-constexpr int kPanelTargets = kP / kPanelTpr;       // targets per thread
-constexpr int kPanelRows = kPanelThreads / kPanelTpr;
-static_assert(kPanelTargets % 4 == 0 && 16 % kPanelTargets == 0, "a thread's targets are whole float4s within a block");
-constexpr int kPanelSmem = (kP * kP + 128 + kPanelRows * (kP + 1)) * 4 + kPanelRows * (kP + 4);
+constexpr int64_t kPanelWideRows = 8192;            // below this many rows: 16 threads per row
+template <int TPR>
+__host__ __device__ constexpr int panel_rows() {
+    return kPanelThreads / TPR;
+}
+template <int TPR>
+__host__ __device__ constexpr int panel_smem() {
+    return (kP * kP + 128 + 2 * panel_rows<TPR>() * (kP + 1)) * 4 + panel_rows<TPR>() * (kP + 4) * 2;
+}
 
-template <int DT>
+template <int DT, int TPR>
 __global__ void __launch_bounds__(kPanelThreads) panel_kernel(LdlqParams p, int64_t k0, int P, float* EpT) {
+    constexpr int kPanelTpr = TPR;                    // threads per row
+    constexpr int kPanelTargets = kP / TPR;           // targets per thread
+    constexpr int kPanelRows = panel_rows<TPR>();
+    static_assert(kPanelTargets % 4 == 0 && 16 % kPanelTargets == 0, "a thread's targets are whole float4s in a block");
     extern __shared__ __align__(16) float dsm[];
     float (*up)[kP] = reinterpret_cast<float (*)[kP]>(dsm);                    // [kP][kP]
     float* rtab = dsm + kP * kP;                                               // [128]
-    float (*wsm)[kP + 1] = reinterpret_cast<float (*)[kP + 1]>(rtab + 128);    // [kPanelRows][kP + 1]
-    uint8_t (*csm)[kP + 4] = reinterpret_cast<uint8_t (*)[kP + 4]>(wsm + kPanelRows);
+    float (*wsm)[kP + 1] = reinterpret_cast<float (*)[kP + 1]>(rtab + 128);    // [kPanelRows][kP + 1] weights
+    float (*rsm)[kP + 1] = wsm + kPanelRows;                                   // fl(1/v) of the element's code, or 0
+    uint16_t (*vsm)[kP + 4] = reinterpret_cast<uint16_t (*)[kP + 4]>(rsm + kPanelRows);   // f16 bits of v
     for (int e = threadIdx.x; e < kP * kP; e += blockDim.x) {
         const int s = e / kP, c = e % kP;
         up[s][c] = (s < c && c < P) ? p.U[(k0 + s) * p.n + k0 + c] : 0.0f;
     }
     for (int c = threadIdx.x; c < 128; c += blockDim.x)
         rtab[c] = (c >= 1 && c <= 126) ? __frcp_rn(f16bits_to_f32(e4m3_to_f16bits((uint32_t)c))) : 0.0f;
+    __syncthreads();                                  // rtab before the row blocks read it
     const float S = __ldg(p.S);
     const float Einv = __frcp_rn(S);
     const bool usable = (S > 0.0f) && isfinite(S) && isfinite(Einv);
     const float E = usable ? Einv : 1.0f;
+    const float Sq = usable ? S : 0.0f;               // an unusable S reconstructs zeros (q is a signed zero then)
     const int lane = threadIdx.x & 31;
     const int kq = threadIdx.x % kPanelTpr;           // this thread's share of the columns
     const int rr = threadIdx.x / kPanelTpr;           // row within the CTA's block
     for (int64_t rb = (int64_t)blockIdx.x * kPanelRows; rb < p.rows; rb += (int64_t)gridDim.x * kPanelRows) {
-        __syncthreads();                              // previous row block done with wsm/csm
+        __syncthreads();                              // rtab written / previous row block done with the row arrays
         {
             float4 wv[kPanelRows * kP / 4 / kPanelThreads];
             uint32_t cv[kPanelRows * kP / 4 / kPanelThreads];
@@ -503,11 +515,15 @@ __global__ void __launch_bounds__(kPanelThreads) panel_kernel(LdlqParams p, int6
 #pragma unroll
             for (int u = 0; u < kPanelRows * kP / 4 / kPanelThreads; u++) {
                 const int e = threadIdx.x + kPanelThreads * u, row = e / (kP / 4), j = 4 * (e % (kP / 4));
-                wsm[row][j] = wv[u].x;
-                wsm[row][j + 1] = wv[u].y;
-                wsm[row][j + 2] = wv[u].z;
-                wsm[row][j + 3] = wv[u].w;
-                *reinterpret_cast<uint32_t*>(&csm[row][j]) = cv[u];
+                const float wq[4] = {wv[u].x, wv[u].y, wv[u].z, wv[u].w};
+#pragma unroll
+                for (int q = 0; q < 4; q++) {
+                    const uint32_t cs = (cv[u] >> (8 * q)) & 0xFFu;
+                    wsm[row][j + q] = wq[q];
+                    // an unusable S or a zero code: r = 0 turns every target into a signed zero
+                    rsm[row][j + q] = usable ? rtab[cs & 127u] : 0.0f;
+                    vsm[row][j + q] = e4m3_to_f16bits(cs);
+                }
             }
         }
         __syncthreads();
@@ -527,34 +543,27 @@ __global__ void __launch_bounds__(kPanelThreads) panel_kernel(LdlqParams p, int6
         uint32_t packed[kPanelTargets / 4] = {};
 #pragma unroll 1
         for (int kb = 0; kb < P / kPanelTargets; kb++) {   // the share whose columns are walked now
-            const bool owner = kq == kb;
+            const bool own = kq == kb && active;
             const int src = (lane & ~(kPanelTpr - 1)) | kb;
 #pragma unroll
             for (int j = 0; j < kPanelTargets; j++) {
                 const int s = kPanelTargets * kb + j;
+                // the column's operands do not depend on the targets: loaded ahead of the chain
+                const float rs = rsm[rr][s], ws = wsm[rr][s];
+                const uint16_t vh = vsm[rr][s];
                 float e = 0.0f;
-                if (owner && active) {
-                    const int cs = csm[rr][s];
-                    const float y = usable ? __fmul_rn(t[j], E) : t[j];
-                    uint32_t nib;
-                    float val;
-                    if (y == 0.0f) {
-                        nib = 0;
-                        val = 0.0f;
-                    } else if (!usable || cs == 0) {
-                        nib = signbit(y) ? 8u : 0u;
-                        val = signbit(y) ? -0.0f : 0.0f;
-                    } else {
-                        const float tq = __fmul_rn(y, rtab[cs]);
-                        nib = e2m1x2(tq, 0.0f) & 0xFu;
-                        uint32_t h2;
-                        asm("{\n\t.reg .b8 b;\n\tcvt.u8.u32 b, %1;\n\tcvt.rn.f16x2.e2m1x2 %0, b;\n\t}"
-                            : "=r"(h2) : "r"(nib));
-                        const float qv = f16bits_to_f32((uint16_t)(h2 & 0xFFFFu));
-                        const float v = f16bits_to_f32(e4m3_to_f16bits((uint32_t)cs));
-                        val = __fmul_rn(__fmul_rn(qv, v), S);
-                    }
-                    e = __fsub_rn(wsm[rr][s], val);
+                if (own) {
+                    // What = fl(fl(q v) S) with q = RNE_E2M1(fl(y r)), y = fl(t E); q v is
+                    // exact, formed by one mixed fma with a +0 addend (a zero q gives +0)
+                    const float y = __fmul_rn(t[j], E);
+                    uint32_t nib = e2m1x2(__fmul_rn(y, rs), 0.0f) & 0xFu;
+                    float qv;
+                    asm("{\n\t.reg .b8 b;\n\t.reg .b32 h2;\n\t.reg .b16 ql, qh;\n\t"
+                        "cvt.u8.u32 b, %1;\n\tcvt.rn.f16x2.e2m1x2 h2, b;\n\tmov.b32 {ql, qh}, h2;\n\t"
+                        "fma.rn.f32.f16 %0, ql, %2, %3;\n\t}"
+                        : "=f"(qv) : "r"(nib), "h"(vh), "f"(0.0f));
+                    if (y == 0.0f) nib = 0;                // an exactly zero target takes the +0 code
+                    e = __fsub_rn(ws, __fmul_rn(qv, Sq));
                     packed[j / 4] |= nib << (8 * (j % 4));
                     EpT[(int64_t)s * p.rows + r] = e;
                 }
@@ -736,13 +745,19 @@ cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* 
     e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64 || !attr_set[dev].load(std::memory_order_acquire)) {
-        e = cudaFuncSetAttribute(panel_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPanelSmem);
+        e = cudaFuncSetAttribute(panel_kernel<0, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, panel_smem<8>());
         if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(panel_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPanelSmem);
+            e = cudaFuncSetAttribute(panel_kernel<1, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, panel_smem<8>());
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(panel_kernel<0, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize, panel_smem<16>());
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(panel_kernel<1, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize, panel_smem<16>());
         if (e != cudaSuccess) return e;
         if (dev >= 0 && dev < 64) attr_set[dev].store(true, std::memory_order_release);
     }
-    const unsigned pg = (unsigned)imin64((p.rows + kPanelRows - 1) / kPanelRows, (int64_t)sms * 16);
+    const bool wide = p.rows < kPanelWideRows;
+    const int prow = wide ? panel_rows<16>() : panel_rows<8>();
+    const unsigned pg = (unsigned)imin64((p.rows + prow - 1) / prow, (int64_t)sms * 16);
     LookAhead* la = nullptr;
     std::unique_lock<std::mutex> lock;
     e = lookahead_for_current_device(&la, &lock);
@@ -758,10 +773,13 @@ cudaError_t launch_ldlq_quantize(LdlqParams p, int dtype, uint8_t* codes, void* 
         for (int64_t k0 = s0; k0 < s0 + span; k0 += kP) {
             const int P = (int)imin64(kP, s0 + span - k0);
             float* Ek = EpT + (k0 - s0) * p.rows;
-            if (dtype == 0)
-                panel_kernel<0><<<pg, kPanelThreads, kPanelSmem, c>>>(p, k0, P, Ek);
-            else
-                panel_kernel<1><<<pg, kPanelThreads, kPanelSmem, c>>>(p, k0, P, Ek);
+            if (wide) {
+                if (dtype == 0) panel_kernel<0, 16><<<pg, kPanelThreads, panel_smem<16>(), c>>>(p, k0, P, Ek);
+                else panel_kernel<1, 16><<<pg, kPanelThreads, panel_smem<16>(), c>>>(p, k0, P, Ek);
+            } else {
+                if (dtype == 0) panel_kernel<0, 8><<<pg, kPanelThreads, panel_smem<8>(), c>>>(p, k0, P, Ek);
+                else panel_kernel<1, 8><<<pg, kPanelThreads, panel_smem<8>(), c>>>(p, k0, P, Ek);
+            }
             e = cudaGetLastError();
             if (e != cudaSuccess) return e;
             const int64_t rest_in = s0 + span - (k0 + P);
