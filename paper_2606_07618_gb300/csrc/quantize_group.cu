@@ -48,6 +48,9 @@ constexpr unsigned long long kGroupWaitNs = 1000000000ull;   // give up a wait f
 #ifndef NVFP4_GROUP_MINB
 #define NVFP4_GROUP_MINB 2
 #endif
+#ifndef NVFP4_GROUP_MINB_MSE
+#define NVFP4_GROUP_MINB_MSE 3
+#endif
 
 __device__ __forceinline__ unsigned long long global_ns() {
     unsigned long long t;
@@ -302,13 +305,13 @@ __device__ __forceinline__ int tensor_at(const GroupParams& p, int t, int64_t se
 // a grid barrier and sweeps with the same 8 warps (phase 2, FP32-bound).
 // AbsMax is HBM-bound in both phases: it is held to 64 registers (4 CTAs per
 // SM, 8 loads in flight per lane in phase 1) for more loads in flight.
-template <int METHOD>
+template <int METHOD, int OBJ>
 constexpr int group_min_blocks() {
-    return METHOD == 1 ? 4 : NVFP4_GROUP_MINB;
+    return METHOD == 1 ? 4 : (OBJ == 0 ? NVFP4_GROUP_MINB_MSE : NVFP4_GROUP_MINB);
 }
 
 template <int DT, int METHOD, int OBJ, int BLOCK, int DYN>
-__global__ void __launch_bounds__(kSweepThreads, group_min_blocks<METHOD>())
+__global__ void __launch_bounds__(kSweepThreads, group_min_blocks<METHOD, OBJ>())
     quantize_group_kernel(const __grid_constant__ GroupParams p) {
     constexpr int SW = kSweepThreads;
     static_assert(SW == kGroupCtaSegments, "host padding unit");
