@@ -149,6 +149,29 @@ def test_ldlq_conditional_parity_small(B, rows, cols, block, dtype):
         assert lg < lr
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_ldlq_tall_weight(B, dtype):
+    """8200 rows (taller weights take the panel walk with eight threads per row,
+    and 8200 is not a multiple of its 16-row CTA): every element checked."""
+    rows, cols = 8200, 192
+    W64, H = rand_problem(rows, cols, 91)
+    Wt = torch.from_numpy(W64.astype(np.float32)).to(dtype)
+    W = Wt.float().numpy().astype(np.float64)
+    H = H.astype(np.float32).astype(np.float64)
+    S, sf = fixed_scales(W, H, 16)
+    perm, U, D, st = prepare(B, H)
+    assert st == 0
+    codes, st = quantize(B, Wt.to(DEV), S, sf, perm, U, 16)
+    assert st == 0
+    bad, exempt, total, first = conditional_parity(W, S, sf, 16, perm.cpu().numpy().astype(np.int64),
+                                                   U.double().cpu().numpy(), codes)
+    assert bad == 0 and first == 0
+    assert exempt <= total // 200
+    ref = L.ldlq(W, H, S, sf, 16)
+    agree = float(np.mean(unpack(codes) == ref["nib"]))
+    assert agree >= 0.99, agree
+
+
 def test_ldlq_full_size_sampled_rows(B):
     """A 4096 x 4096 weight (q/o projection shape) with a low-rank-plus-diagonal
     Hessian of heavy-tailed channel scales; 48 sampled rows checked in float64."""
