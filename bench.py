@@ -265,8 +265,8 @@ def run_gpu(args, rank, world):
     hbm_peak, peak_kind = peaks()
 
     # The step: one grouped launch over both matrices that reduces each one's
-    # global scale in the same launch (a ninth warp per CTA streams the
-    # reductions while the other eight sweep) and sweeps every block.
+    # global scale in the same launch (every warp folds its share of both
+    # matrices, then a grid barrier) and sweeps every block.
     def step(events=None):
         if events is not None:
             events[0].record(stream)
@@ -615,7 +615,8 @@ def config_dict(wl, world):
             "scale_layouts": "linear+swizzled",
             "parallelism": f"replicas{world}" if world > 1 else "single-gpu",
             "l2": "no flush: each step streams the 968 MB of inputs (> 129 MB L2) twice, once for the global scales "
-                  "and once for the sweep; inside the one launch matrix 2's scale is reduced while matrix 1 is swept"}
+                  "and once for the sweep; inside the one launch both scales are reduced first, then every CTA "
+                  "passes a grid barrier and sweeps"}
 
 
 def run_kernel_case(args):
