@@ -650,6 +650,8 @@ def run_kernel_case(args):
         "four_six": lambda: B.four_over_six_quantize(x, args.block, S, 1, w, 0, o["codes"], o["sf_linear"],
                                                      o["sf_swizzled"]),
         "dequant": lambda: B.nvfp4_dequantize(o["codes"], o["sf_linear"], 1, S, args.rows, args.cols, args.block, dq),
+        "dequant_swizzled": lambda: B.nvfp4_dequantize(o["codes"], o["sf_swizzled"], B.NVFP4_SF_SWIZZLED, S, args.rows,
+                                                       args.cols, args.block, dq),
         "amax": lambda: B.nvfp4_global_scale(x, 256.0, S, None, ws),
         "mse_two_launch": lambda: (B.nvfp4_global_scale(x, 256.0, S, None, ws),
                                    B.scalesweep_quantize(x, args.block, S, 0, None, 0, *win, o["codes"],
@@ -985,7 +987,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-rows", type=int, default=64)
     ap.add_argument("--kernel-case", default=None,
-                    choices=["sweep_wmse", "sweep_mse", "absmax", "four_six", "dequant", "amax", "mse_two_launch",
+                    choices=["sweep_wmse", "sweep_mse", "absmax", "four_six", "dequant", "dequant_swizzled", "amax",
+                             "mse_two_launch",
                              "sweep_wmse_group", "wmse_group_dynamic", "group_layer", "group_layer_static",
                              "sweep_wmse_tight", "sweep_mse_tight",
                              "layer_per_tensor_static", "group_layer_linear", "group_layer_static_linear",
