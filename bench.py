@@ -264,9 +264,11 @@ def run_gpu(args, rank, world):
     nsm = torch.cuda.get_device_properties(dev).multi_processor_count
     hbm_peak, peak_kind = peaks()
 
-    # The step: one grouped launch over both matrices that reduces each one's
-    # global scale in the same launch (every warp folds its share of both
-    # matrices, then a grid barrier) and sweeps every block.
+    # The step: one grouped call over both matrices that reduces each one's
+    # global scale on the device and sweeps every block.  At this size the
+    # library runs its pipelined schedule: the larger matrix's reduction, its
+    # sweep with the other matrix's reduction running beside it on the
+    # registers the sweep leaves free, then the other matrix's sweep.
     def step(events=None):
         if events is not None:
             events[0].record(stream)
@@ -274,7 +276,9 @@ def run_gpu(args, rank, world):
         if events is not None:
             events[1].record(stream)
 
-    launches_per_step = 1   # the grouped kernel (the workspace reset is a memset; these shapes need no pad kernel)
+    # two reductions and two sweeps (the workspace reset is a memset; these
+    # shapes need no swizzle pad kernel)
+    launches_per_step = 4 if st.pipelined else 1
 
     for _ in range(args.warmup):
         step()
@@ -299,7 +303,9 @@ def run_gpu(args, rank, world):
     value = world * total / (ms_step * 1e-3) / 1e9
     assert int(st.status.item()) == 0, "non-finite input detected"
 
-    # ---- roofline of the dominant (only) kernel, from the per-step events
+    # ---- roofline of the step's kernels as one unit, from the per-step events
+    # (the two reductions run beside the sweeps, so the call is the unit a
+    # CUDA event can bracket without breaking the overlap)
     clk_sum = clk.summary()
     sm_mhz = clk_sum["sm_mhz"] or clk_sum["sm_max_mhz"] or 2070
     alu_peak = nsm * 128 * sm_mhz * 1e6
@@ -313,16 +319,23 @@ def run_gpu(args, rank, world):
     gbs, hfrac, tops, afrac = fracs(wl, xs, kern_ms)
     roofline = {"bound": "alu", "achieved": tops, "peak": round(alu_peak / 1e12, 3), "unit": "Tops/s",
                 "frac": afrac, "traffic": None,
-                "kernel": f"quantize_group_kernel<bf16,ScaleSweep,WMSE,block {wl.block},dynamic S> "
-                          f"({len(xs)} tensors, one launch per step)",
+                "kernel": (f"quantize_group_kernel<bf16,ScaleSweep,WMSE,block {wl.block},pipelined S> x2 with "
+                           f"group_reduce_kernel x2 beside them ({len(xs)} tensors, one call per step)")
+                if st.pipelined else
+                f"quantize_group_kernel<bf16,ScaleSweep,WMSE,block {wl.block},dynamic S> "
+                f"({len(xs)} tensors, one launch per step)",
                 "peak_note": f"{nsm} SMs x 128 FP32 lanes x median SM clock {sm_mhz} MHz "
                              f"(of measured clock; the work is {alu_ops_per_elem(wl)} FP32 ops per element: "
                              f"{candidates(wl)} candidates x 4)",
                 "hbm": {"achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": hfrac, "peak_kind": peak_kind,
                         "bytes": round(hbm_bytes(wl, xs)), "bytes_per_elem": round(hbm_bytes(wl, xs) / total, 4)},
                 "launch_ms": round(kern_ms, 4),
-                "launch_note": "events around the call: the 256-byte workspace memset and the kernel"}
-    roofline["traffic"] = traffic_per_launch("quantize_group_kernel_qwen72b_traffic.json", total)
+                "launch_note": "events around the call: the 256-byte workspace memset and the "
+                               + ("four launches" if st.pipelined else "kernel")}
+    # DRAM bytes of the step's launches from one ncu capture (null for the
+    # two-phase schedule, which has no current record)
+    roofline["traffic"] = traffic_per_launch("quantize_group_pipelined_qwen72b_traffic.json", total) \
+        if st.pipelined else None
 
     reps = max(3, min(20, args.steps))
     flush = L2Flush(dev)
@@ -366,6 +379,10 @@ def run_gpu(args, rank, world):
         B.scalesweep_quantize_group(st_static.desc, st_static.dtype, B.NVFP4_OBJ_WMSE, 0.0, S_fixed, None, None,
                                     stream=stream, block=wl.block)
 
+    def two_phase():
+        B.scalesweep_quantize_group(st.desc, st.dtype, B.NVFP4_OBJ_WMSE, wl.fp8_div, st.S, st.status, st.workspace,
+                                    stream=stream, block=wl.block, schedule=B.NVFP4_GROUP_SCHEDULE_TWO_PHASE)
+
     def absmax_static():
         B.absmax_quantize_group(st_static.desc, st_static.dtype, 0.0, S_fixed, None, None, stream=stream,
                                 block=wl.block)
@@ -403,6 +420,7 @@ def run_gpu(args, rank, world):
         return dict(value=value, ms_step=ms_step, total=total, roofline=roofline, clocks=clk_sum, legs=None,
                     overhead=None, e2e=None, cpu=None, launches=launches_per_step * args.steps, wl=wl)
     t_gs = time_calls(static_sweep, reps, stream)
+    t_2p = time_calls(two_phase, reps, stream)
     t_as = time_calls(absmax_static, reps, stream)
     t_pt = time_calls(per_tensor_launches, reps, stream)
     t_46 = time_calls(four_six, reps, stream)
@@ -412,6 +430,7 @@ def run_gpu(args, rank, world):
                                                                              stream)
     legs[WORKLOAD + " (headline) static scales"] = {
         "scalesweep_grouped_static": {"ms": round(t_gs, 4), "gelem_s": gel(t_gs)},
+        "scalesweep_grouped_dynamic_two_phase_schedule": {"ms": round(t_2p, 4), "gelem_s": gel(t_2p)},
         "absmax_grouped_static": {"ms": round(t_as, 4), "gelem_s": gel(t_as)},
         "per_tensor_global_scale_then_sweep": {"ms": round(t_pt, 4), "gelem_s": gel(t_pt)},
         "four_over_six_wmse_per_tensor": {"ms": round(t_46, 4), "gelem_s": gel(t_46)},
@@ -611,12 +630,12 @@ def config_dict(wl, world):
     return {"workload": "qwen2.5-72b-shaped-weights-wmse-block16",
             "tensors": {t.name: [t.rows, t.cols] for t in wl.tensors},
             "elements": wl.numel, "input": "bf16", "block": wl.block, "objective": wl.objective,
-            "global_scale": f"amax/(6*{int(wl.fp8_div)}) computed every step, in the launch",
+            "global_scale": f"amax/(6*{int(wl.fp8_div)}) computed on the device every step, in the call",
             "scale_layouts": "linear+swizzled",
             "parallelism": f"replicas{world}" if world > 1 else "single-gpu",
             "l2": "no flush: each step streams the 968 MB of inputs (> 129 MB L2) twice, once for the global scales "
-                  "and once for the sweep; inside the one launch both scales are reduced first, then every CTA "
-                  "passes a grid barrier and sweeps"}
+                  "and once for the sweep (the pipelined schedule: the larger matrix's reduction, then its sweep "
+                  "with the other matrix's reduction beside it, then the other matrix's sweep)"}
 
 
 def run_kernel_case(args):

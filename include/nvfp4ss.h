@@ -211,26 +211,27 @@ size_t scalesweep_quantize_group_workspace(void);
 
 /*
  * ScaleSweep quantisation of `count` tensors (1..NVFP4_GROUP_MAX, e.g. all
- * linear weights of one transformer layer) in one launch: for every tensor the
+ * linear weights of one transformer layer) in one call: for every tensor the
  * result of scalesweep_quantize with the same block and the default window
  * ([-3, 7] MSE with block 16, [-8, 7] otherwise, Sec. 4.2.2), bit for bit.  The
- * segments of all tensors are walked by one grid, so the call has a single
- * launch tail instead of one per tensor.
+ * segments of all tensors are walked by one grid (with static scales, one
+ * launch), so the call has a single launch tail instead of one per tensor.
  *   tensors     host array of `count` descriptors, read during the call only.
  *   dt, obj     input type and objective, shared by all tensors.
  *   block       16, 32 or 64, shared by all tensors (every cols % block == 0);
  *               sf_swizzled only with block 16.
  *   fp8_div     0: static global scales, S[i] is read for tensor i.
  *               > 0: per-call (dynamic) global scales, S[i] = fl32(amax_i /
- *               fl32(6*fp8_div)) over tensor i (Sec. 4.2.1) is computed in the
- *               same launch and written: every warp first reduces its share of
- *               every tensor, then a grid barrier, then the sweep (cooperative
- *               launch, preceded by a cudaMemsetAsync of the workspace counters).
+ *               fl32(6*fp8_div)) over tensor i (Sec. 4.2.1) is computed on the
+ *               device during the call and written, by the schedule
+ *               NVFP4_GROUP_SCHEDULE_AUTO picks (see
+ *               scalesweep_quantize_group_scheduled); either is preceded by a
+ *               cudaMemsetAsync of the workspace counters.
  *   S           device float[count].
  *   status_dev  optional device int: bit 0 OR-ed in for NaN/inf input (dynamic
- *               only), bit 1 if the grid barrier timed out (about a second; no
- *               outputs are written then -- a resident grid makes this
- *               unreachable in practice).
+ *               only), bit 1 if the two-phase schedule's grid barrier timed out
+ *               (about a second; no outputs are written then -- a resident grid
+ *               makes this unreachable in practice).
  *   workspace   scalesweep_quantize_group_workspace() bytes, 16-byte aligned, no
  *               initialisation (dynamic only; may be NULL for static scales).
  * Outputs must not overlap any input, S, status_dev, the workspace or each
@@ -239,6 +240,41 @@ size_t scalesweep_quantize_group_workspace(void);
 nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt, int block,
                                        nvfp4_objective obj, float fp8_div, float* S, int* status_dev,
                                        void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * How a grouped call with dynamic global scales (fp8_div > 0) orders the
+ * reduction of every tensor's amax and the sweep.  Results are identical, bit
+ * for bit, under every schedule; only the launches and their overlap differ.
+ *   NVFP4_GROUP_SCHEDULE_AUTO       pipelined for a ScaleSweep over at least
+ *                                   two tensors and 2^25 elements, else two-phase.
+ *   NVFP4_GROUP_SCHEDULE_TWO_PHASE  one cooperative launch: every warp reduces
+ *                                   its share of every tensor, a grid barrier
+ *                                   (bounded, status bit 1), then the sweep.
+ *   NVFP4_GROUP_SCHEDULE_PIPELINED  four launches, the last three programmatic
+ *                                   dependent launches: the largest tensor's
+ *                                   reduction, its sweep, the other tensors'
+ *                                   reduction running beside that sweep on the
+ *                                   registers it leaves free, then one grouped
+ *                                   sweep of the other tensors.  The HBM-bound
+ *                                   reductions hide behind the FP32-bound sweep,
+ *                                   except the first.  No device wait is involved.
+ *                                   With one tensor, or for AbsMax, two-phase.
+ */
+typedef enum {
+    NVFP4_GROUP_SCHEDULE_AUTO = 0,
+    NVFP4_GROUP_SCHEDULE_TWO_PHASE = 1,
+    NVFP4_GROUP_SCHEDULE_PIPELINED = 2
+} nvfp4_group_schedule;
+
+/*
+ * scalesweep_quantize_group with an explicit schedule for dynamic global
+ * scales (ignored when fp8_div == 0).  Arguments, outputs and errors as
+ * scalesweep_quantize_group; an unknown schedule is NVFP4_ERR_INVALID_ARG.
+ */
+nvfp4_status scalesweep_quantize_group_scheduled(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt,
+                                                 int block, nvfp4_objective obj, float fp8_div, float* S,
+                                                 int* status_dev, void* workspace, size_t ws_bytes,
+                                                 nvfp4_group_schedule schedule, void* stream);
 
 /*
  * AbsMax quantisation (Sec. 3.2, as absmax_quantize) of `count` tensors in one

@@ -34,6 +34,7 @@ class Nvfp4Error(RuntimeError):
 _lib = None
 
 NVFP4_GROUP_MAX = 16
+NVFP4_GROUP_SCHEDULE_AUTO, NVFP4_GROUP_SCHEDULE_TWO_PHASE, NVFP4_GROUP_SCHEDULE_PIPELINED = 0, 1, 2
 
 
 class RowShard(ctypes.Structure):
@@ -77,6 +78,8 @@ def lib() -> ctypes.CDLL:
         L.absmax_quantize_dynamic.argtypes = [p, i, i64, i64, i, f, p, p, p, sz, p, p, p, p, p]
         L.scalesweep_quantize_group_workspace.argtypes, L.scalesweep_quantize_group_workspace.restype = [], sz
         L.scalesweep_quantize_group.argtypes = [ctypes.POINTER(GroupTensor), i, i, i, i, f, p, p, p, sz, p]
+        L.scalesweep_quantize_group_scheduled.argtypes = [ctypes.POINTER(GroupTensor), i, i, i, i, f, p, p, p, sz,
+                                                          i, p]
         L.absmax_quantize_group.argtypes = [ctypes.POINTER(GroupTensor), i, i, i, f, p, p, p, sz, p]
         L.nvfp4_selftest_wait_timeout.argtypes = [i, p, i64, i64, p, p, p, sz, p, p, p]
         L.nvfp4_row_shard_layout.argtypes = [i64, i64, i, i, i, ctypes.POINTER(RowShard)]
@@ -88,7 +91,8 @@ def lib() -> ctypes.CDLL:
         for fn in ("nvfp4_global_scale", "nvfp4_global_scale_noalloc", "scalesweep_quantize", "absmax_quantize",
                    "four_over_six_quantize", "nvfp4_dequantize", "scalesweep_quantize_dynamic",
                    "absmax_quantize_dynamic", "nvfp4_optimal_scale", "nvfp4_ldlq_prepare", "ldlq_quantize",
-                   "scalesweep_quantize_group", "absmax_quantize_group", "nvfp4_selftest_wait_timeout",
+                   "scalesweep_quantize_group", "scalesweep_quantize_group_scheduled", "absmax_quantize_group",
+                   "nvfp4_selftest_wait_timeout",
                    "nvfp4_row_shard_layout"):
             getattr(L, fn).restype = i
         _lib = L
@@ -217,13 +221,21 @@ def group_descriptors(xs, ws, w_row_strides, codes, sf_linear, sf_swizzled):
 
 
 def scalesweep_quantize_group(desc, dtype: int, objective: int, fp8_div: float, S, status=None, workspace=None,
-                              stream=None, block: int = 16):
+                              stream=None, block: int = 16, schedule: int | None = None):
     """desc: the array from group_descriptors.  fp8_div 0 reads S[i]; > 0
-    computes and writes S[i] in the launch."""
+    computes and writes S[i] during the call.  schedule None calls
+    scalesweep_quantize_group (the library's choice); an NVFP4_GROUP_SCHEDULE_*
+    value calls scalesweep_quantize_group_scheduled with it."""
     ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
-    rc = lib().scalesweep_quantize_group(desc, len(desc), int(dtype), int(block), int(objective), float(fp8_div),
-                                         _ptr(S), _ptr(status), _ptr(workspace), ws_bytes, _stream(stream))
-    _check("scalesweep_quantize_group", rc)
+    if schedule is None:
+        rc = lib().scalesweep_quantize_group(desc, len(desc), int(dtype), int(block), int(objective), float(fp8_div),
+                                             _ptr(S), _ptr(status), _ptr(workspace), ws_bytes, _stream(stream))
+        _check("scalesweep_quantize_group", rc)
+    else:
+        rc = lib().scalesweep_quantize_group_scheduled(desc, len(desc), int(dtype), int(block), int(objective),
+                                                       float(fp8_div), _ptr(S), _ptr(status), _ptr(workspace),
+                                                       ws_bytes, int(schedule), _stream(stream))
+        _check("scalesweep_quantize_group_scheduled", rc)
 
 
 def absmax_quantize_group(desc, dtype: int, fp8_div: float, S, status=None, workspace=None, stream=None,

@@ -281,8 +281,12 @@ namespace {
 // method 0 ScaleSweep (objective obj), 1 AbsMax (obj ignored: MSE, no weights read).
 nvfp4_status group_common(int method, const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt, int block,
                           nvfp4_objective obj, float fp8_div, float* S, int* status_dev, void* workspace,
-                          size_t ws_bytes, void* stream, unsigned wait_extra) {
+                          size_t ws_bytes, void* stream, unsigned wait_extra,
+                          nvfp4_group_schedule schedule = NVFP4_GROUP_SCHEDULE_AUTO) {
     if (dt != NVFP4_IN_BF16 && dt != NVFP4_IN_F32) return NVFP4_ERR_INVALID_ARG;
+    if (schedule != NVFP4_GROUP_SCHEDULE_AUTO && schedule != NVFP4_GROUP_SCHEDULE_TWO_PHASE &&
+        schedule != NVFP4_GROUP_SCHEDULE_PIPELINED)
+        return NVFP4_ERR_INVALID_ARG;
     if (method == 1) obj = NVFP4_OBJ_MSE;
     if (obj != NVFP4_OBJ_MSE && obj != NVFP4_OBJ_WMSE) return NVFP4_ERR_INVALID_ARG;
     if (!tensors || count < 1 || count > NVFP4_GROUP_MAX || !S) return NVFP4_ERR_INVALID_ARG;
@@ -389,6 +393,10 @@ nvfp4_status group_common(int method, const nvfp4_group_tensor* tensors, int cou
     }
     p.count = count;
     p.dyn = dyn ? 1 : 0;
+    int64_t elements = 0;
+    for (int i = 0; i < count; i++) elements += sh[i].n < kPipelineMinElements ? sh[i].n : kPipelineMinElements;
+    p.pipelined = schedule == NVFP4_GROUP_SCHEDULE_PIPELINED ||
+                  (schedule == NVFP4_GROUP_SCHEDULE_AUTO && count >= 2 && elements >= kPipelineMinElements);
     p.total_seg = seg;
     p.fp8_div = fp8_div;
     p.S = S;
@@ -407,6 +415,14 @@ nvfp4_status scalesweep_quantize_group(const nvfp4_group_tensor* tensors, int co
                                        nvfp4_objective obj, float fp8_div, float* S, int* status_dev,
                                        void* workspace, size_t ws_bytes, void* stream) {
     return group_common(0, tensors, count, dt, block, obj, fp8_div, S, status_dev, workspace, ws_bytes, stream, 0);
+}
+
+nvfp4_status scalesweep_quantize_group_scheduled(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt,
+                                                 int block, nvfp4_objective obj, float fp8_div, float* S,
+                                                 int* status_dev, void* workspace, size_t ws_bytes,
+                                                 nvfp4_group_schedule schedule, void* stream) {
+    return group_common(0, tensors, count, dt, block, obj, fp8_div, S, status_dev, workspace, ws_bytes, stream, 0,
+                        schedule);
 }
 
 nvfp4_status absmax_quantize_group(const nvfp4_group_tensor* tensors, int count, nvfp4_dtype dt, int block,
@@ -428,7 +444,7 @@ nvfp4_status nvfp4_selftest_wait_timeout(int which, const void* x, int64_t rows,
     }
     const nvfp4_group_tensor t{x, rows, cols, nullptr, 0, codes, sf_linear, nullptr};
     return group_common(0, &t, 1, NVFP4_IN_BF16, 16, NVFP4_OBJ_MSE, 256.0f, S, status_dev, workspace, ws_bytes,
-                        stream, 1);
+                        stream, 1, NVFP4_GROUP_SCHEDULE_TWO_PHASE);
 }
 
 nvfp4_status absmax_quantize_dynamic(const void* x, nvfp4_dtype dt, int64_t rows, int64_t cols, int block,

@@ -32,6 +32,7 @@ struct GroupParams {
     GroupTensor t[kGroupMax];  // in processing order
     int count;
     int dyn;                   // 1: S computed in the launch, 0: S read
+    int pipelined;             // dyn only: 1 pipelined schedule, 0 two-phase cooperative launch
     int64_t total_seg;         // end of the concatenated segment space
     float fp8_div;
     float* S;                  // [count] by s_index
@@ -43,6 +44,10 @@ struct GroupParams {
 
 constexpr size_t kGroupWorkspace = 256;   // amax_bits + arrived for kGroupMax tensors
 
+// Groups of at least this many elements (and two tensors) take the pipelined
+// schedule when the caller leaves the choice to the library.
+constexpr int64_t kPipelineMinElements = int64_t(1) << 25;
+
 // Segments a CTA sweeps per iteration; each tensor's segment range in the
 // concatenated index space is padded to a multiple of it, so a CTA never
 // straddles two tensors.
@@ -50,8 +55,9 @@ constexpr int kGroupCtaSegments = 256;
 
 // dtype 0 bf16 / 1 f32; method 0 ScaleSweep / 1 AbsMax; obj 0 MSE / 1 WMSE
 // (ScaleSweep only); block 16/32/64.  Zeroes the workspace counters (dyn),
-// launches the grouped kernel (cooperative when dyn) and the swizzle pad
-// kernels for shapes that need them.
+// launches the grouped kernel (cooperative when dyn; with p.pipelined, a
+// ScaleSweep and at least two tensors, the four launches of the pipelined
+// schedule instead) and the swizzle pad kernels for shapes that need them.
 cudaError_t launch_quantize_group(const GroupParams& p, const int64_t* rows, int dtype, int method, int obj,
                                   int block, int sms, cudaStream_t s);
 

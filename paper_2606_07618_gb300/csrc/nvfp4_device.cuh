@@ -123,6 +123,16 @@ __device__ __forceinline__ uint4 ld_ro16(const void* p) {
     return v;
 }
 
+// Programmatic dependent launch: the running grid lets a kernel launched after
+// it with cudaLaunchAttributeProgrammaticStreamSerialization be scheduled once
+// every CTA of this grid has executed launch_dependents (or exited); that
+// kernel's griddepcontrol.wait returns once this grid has completed and its
+// writes are visible (and at once when it was launched the ordinary way).
+__device__ __forceinline__ void grid_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ float bf16lo(uint32_t u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t u) { return __uint_as_float(u & 0xFFFF0000u); }
 

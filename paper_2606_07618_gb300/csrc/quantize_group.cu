@@ -18,7 +18,9 @@
 // and both scale layouts; blocks of 32/64 are 2/4 lanes combined by
 // xor-shuffles (a CTA's 256 segments always hold whole blocks).
 //
-// In-launch global scales (cooperative launch, two phases).  Phase 1: every
+// In-launch global scales, two schedules with bit-identical results.
+//
+// Two-phase (one cooperative launch).  Phase 1: every
 // warp of the grid folds max |x| over its share of every tensor (16 loads in
 // flight per lane, on the integer pipe: with the sign bit cleared the unsigned
 // order of bf16/fp32 bit patterns is the order of the magnitudes) and
@@ -33,6 +35,15 @@
 // registers and interfered with the sweep's loads; on the two 242M-element
 // matrices of the Qwen2.5-72B shapes, where only half the data can overlap
 // at all, it measured 1.674 ms against 1.409 ms for the sweep alone.)
+//
+// Pipelined (four launches, launch_group_pipelined).  The reduction runs as a
+// separate kernel of 32-register threads, which the SM holds beside the sweep
+// CTAs on the registers they leave free: the largest tensor is reduced, then
+// swept while the other tensors are reduced beside it, then the others are
+// swept.  Only the first reduction is exposed.  On the two Qwen2.5-72B-shaped
+// matrices (WMSE) 1.506-1.512 ms per call against 1.568-1.573 ms two-phase and
+// 1.406-1.411 ms with static scales; on the Llama-3-8B layer 0.681 against
+// 0.735 (static 0.643).
 #include <atomic>
 
 #include "group_kernels.h"
@@ -44,6 +55,8 @@ namespace {
 
 constexpr int kSweepThreads = 256;                          // sweep threads per CTA
 constexpr int kAmaxInFlight = 16;                           // 16-byte loads in flight per reduction lane
+constexpr int kReduceThreads = 128;                         // pipelined schedule: reduction CTA size
+constexpr int kReduceInFlight = 4;                          // and its loads in flight per lane (32 registers)
 constexpr unsigned long long kGroupWaitNs = 1000000000ull;   // give up a wait for a scale after 1 s
 #ifndef NVFP4_GROUP_MINB
 #define NVFP4_GROUP_MINB 2
@@ -51,6 +64,14 @@ constexpr unsigned long long kGroupWaitNs = 1000000000ull;   // give up a wait f
 #ifndef NVFP4_GROUP_MINB_MSE
 #define NVFP4_GROUP_MINB_MSE 3
 #endif
+// Pipelined schedule: sweep CTAs per SM beside which the other tensors'
+// reduction runs when those tensors hold more than half the first one's bytes.
+// The MSE sweep could hold 3 CTAs per SM, which leaves the reduction one warp
+// per scheduler: on the two Qwen2.5-72B-shaped matrices (MSE) that reduction
+// then outlasts the sweep it should hide behind (0.964 ms per call against
+// 0.890 ms with 2 CTAs); on K, V, Q (the rest is half of Q) 3 CTAs are faster
+// (0.751 against 0.765-0.774 ms).
+constexpr int kPipeSweepCtas = 2;
 
 __device__ __forceinline__ unsigned long long global_ns() {
     unsigned long long t;
@@ -111,11 +132,11 @@ __device__ __noinline__ float rescan_share(const uint4* xv, int64_t nvec, int64_
 // max, so S matches the two-launch path bit for bit, and sets status bit 0
 // for NaN/inf.  Each warp's atomics are fenced before the CTA arrives at the
 // grid barrier.
-template <int DT, int INFLIGHT>
+template <int DT, int INFLIGHT, int THREADS = kSweepThreads>
 __device__ __forceinline__ void reduce_all(const GroupParams& p) {
     const int lane = threadIdx.x & 31;
-    const int64_t W = (int64_t)gridDim.x * (kSweepThreads / 32);
-    const int64_t w = (int64_t)blockIdx.x * (kSweepThreads / 32) + (threadIdx.x >> 5);
+    const int64_t W = (int64_t)gridDim.x * (THREADS / 32);
+    const int64_t w = (int64_t)blockIdx.x * (THREADS / 32) + (threadIdx.x >> 5);
     const int64_t step = W * 32, first = w * 32 + lane;
     bool any_bad = false;
     for (int a = 0; a < p.count; a++) {
@@ -178,6 +199,30 @@ __device__ __forceinline__ bool grid_barrier(const GroupParams& p) {
     }
     __syncthreads();
     return !s_timeout;
+}
+
+// Pipelined schedule of in-launch global scales: the reduction of one set of
+// tensors as a kernel of its own, with 32 registers per thread so that it fits
+// beside the sweep kernel's CTAs on an SM.  Every warp folds its share of
+// every tensor of p (as phase 1 of the two-phase launch), then the last CTA to
+// arrive (a ticket counter in the caller's workspace, zeroed before the
+// launch) writes S[t] = fl(amax_t / fl(6 D)).  Nothing waits on another CTA.
+// Launched as a programmatic dependent of a sweep kernel, the grid is
+// scheduled once every CTA of that sweep is resident, reads only its own
+// tensors, and ends with griddepcontrol.wait, so it completes (and the next
+// sweep, which waits for it, starts) only after that sweep has completed.
+template <int DT>
+__global__ void __launch_bounds__(kReduceThreads, 2048 / kReduceThreads)
+    group_reduce_kernel(const __grid_constant__ GroupParams p, unsigned* ticket) {
+    reduce_all<DT, kReduceInFlight, kReduceThreads>(p);
+    __syncthreads();                                 // every warp's atomics are fenced
+    if (threadIdx.x == 0 && atom_add_acq_rel(ticket, 1u) == gridDim.x - 1) {
+        for (int a = 0; a < p.count; a++)            // the last CTA sees every CTA's maxima
+            p.S[p.t[a].s_index] =
+                __fdiv_rn(__uint_as_float(ld_relaxed_u32(p.amax_bits + a)), __fmul_rn(6.0f, p.fp8_div));
+    }
+    grid_launch_dependents();
+    grid_dependency_wait();
 }
 
 // One 16-element segment of the grid-stride loop: ScaleSweep (METHOD 0,
@@ -305,6 +350,8 @@ __device__ __forceinline__ int tensor_at(const GroupParams& p, int t, int64_t se
 // a grid barrier and sweeps with the same 8 warps (phase 2, FP32-bound).
 // AbsMax is HBM-bound in both phases: it is held to 64 registers (4 CTAs per
 // SM, 8 loads in flight per lane in phase 1) for more loads in flight.
+// DYN = 2: the pipelined schedule's sweep, scales from the reduction grid
+// launched before it.
 template <int METHOD, int OBJ>
 constexpr int group_min_blocks() {
     return METHOD == 1 ? 4 : (OBJ == 0 ? NVFP4_GROUP_MINB_MSE : NVFP4_GROUP_MINB);
@@ -317,12 +364,18 @@ __global__ void __launch_bounds__(kSweepThreads, group_min_blocks<METHOD, OBJ>()
     static_assert(SW == kGroupCtaSegments, "host padding unit");
     __shared__ Cand tab[kTabN];
     build_table(tab);
-    if (DYN) {
+    if (DYN == 1) {
         reduce_all<DT, METHOD == 1 ? 8 : kAmaxInFlight>(p);
         if (!grid_barrier(p)) return;
         if (blockIdx.x == 0 && (int)threadIdx.x < p.count)        // publish every tensor's S once
             p.S[p.t[threadIdx.x].s_index] =
                 __fdiv_rn(__uint_as_float(ld_relaxed_u32(p.amax_bits + threadIdx.x)), __fmul_rn(6.0f, p.fp8_div));
+    } else if (DYN == 2) {
+        // pipelined schedule: the scales come from the reduction grid launched
+        // before this one; once every CTA is resident the next reduction grid
+        // may be scheduled beside it
+        grid_dependency_wait();
+        grid_launch_dependents();
     }
     __syncthreads();
 
@@ -345,8 +398,10 @@ __global__ void __launch_bounds__(kSweepThreads, group_min_blocks<METHOD, OBJ>()
 
     while (cbase < total) {
         // entering tensor t: its global scale
-        const float S = DYN ? __fdiv_rn(__uint_as_float(ld_relaxed_u32(p.amax_bits + t)), __fmul_rn(6.0f, p.fp8_div))
-                            : __ldg(p.S + p.t[t].s_index);
+        const float S =
+            DYN == 1 ? __fdiv_rn(__uint_as_float(ld_relaxed_u32(p.amax_bits + t)), __fmul_rn(6.0f, p.fp8_div))
+            : DYN == 2 ? __uint_as_float(ld_relaxed_u32(reinterpret_cast<const unsigned*>(p.S + p.t[t].s_index)))
+                       : __ldg(p.S + p.t[t].s_index);
         float E = __frcp_rn(S);
         const bool usable = (S > 0.0f) && isfinite(S) && isfinite(E);
         if (!usable) E = 1.0f;
@@ -377,19 +432,23 @@ __global__ void __launch_bounds__(kSweepThreads, group_min_blocks<METHOD, OBJ>()
 
 namespace {
 
+// Resident sweep CTAs per SM and the grid of one sweep launch over p: the
+// whole segment space, capped at the resident maximum (every wait can then
+// complete); for WMSE up to 1/32 fewer CTAs if that makes the CTA stride a
+// multiple of more tensors' segments per row (lanes then keep their weights).
 template <int DT, int METHOD, int OBJ, int BLOCK, int DYN>
-cudaError_t launch_group(const GroupParams& p, int sms, cudaStream_t s) {
-    constexpr int SW = kSweepThreads, threads = kSweepThreads;
+int64_t sweep_grid(const GroupParams& p, int sms, int* per_sm, int max_per_sm = 0) {
+    constexpr int SW = kSweepThreads;
     constexpr int SEGS = BLOCK / 16;
     static std::atomic<int> occ_cache[kOccDevices];
-    const int64_t cap = (int64_t)sms *
-                        occupancy_per_sm(occ_cache, quantize_group_kernel<DT, METHOD, OBJ, BLOCK, DYN>, threads);
+    int occ = occupancy_per_sm(occ_cache, quantize_group_kernel<DT, METHOD, OBJ, BLOCK, DYN>, SW);
+    if (max_per_sm > 0 && occ > max_per_sm) occ = max_per_sm;
+    if (per_sm) *per_sm = occ;
+    const int64_t cap = (int64_t)sms * occ;
     int64_t grid = (p.total_seg + SW - 1) / SW;
     if (grid > cap) {
-        grid = cap;                                              // resident grid: every wait can complete
+        grid = cap;
         if (METHOD == 0 && OBJ == 1) {
-            // Up to 1/32 fewer CTAs if that makes the CTA stride a multiple of
-            // more tensors' segments per row (lanes then keep their weights).
             auto covered = [&](int64_t g) {
                 int64_t c = 0;
                 for (int i = 0; i < p.count; i++)
@@ -408,29 +467,119 @@ cudaError_t launch_group(const GroupParams& p, int sms, cudaStream_t s) {
             grid = best;
         }
     }
-    if (grid < 1) grid = 1;
+    return grid < 1 ? 1 : grid;
+}
+
+template <int DT, int METHOD, int OBJ, int BLOCK, int DYN>
+cudaError_t launch_group(const GroupParams& p, int sms, cudaStream_t s) {
+    const int64_t grid = sweep_grid<DT, METHOD, OBJ, BLOCK, DYN>(p, sms, nullptr);
     if (DYN) {
         cudaError_t e = cudaMemsetAsync(p.amax_bits, 0, kGroupWorkspace, s);
         if (e != cudaSuccess) return e;
         void* args[] = {(void*)&p};
         return cudaLaunchCooperativeKernel((const void*)quantize_group_kernel<DT, METHOD, OBJ, BLOCK, 1>,
-                                           dim3((unsigned)grid), dim3(threads), args, 0, s);
+                                           dim3((unsigned)grid), dim3(kSweepThreads), args, 0, s);
     }
-    quantize_group_kernel<DT, METHOD, OBJ, BLOCK, 0><<<(unsigned)grid, threads, 0, s>>>(p);
+    quantize_group_kernel<DT, METHOD, OBJ, BLOCK, 0><<<(unsigned)grid, kSweepThreads, 0, s>>>(p);
     return cudaGetLastError();
 }
 
+// Launch of `kernel` on `s` as a programmatic dependent of the kernel before
+// it on the stream.
+template <typename... Args>
+cudaError_t launch_dependent(void (*kernel)(Args...), int64_t grid, int threads, cudaStream_t s, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3((unsigned)threads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
+// The tensors p.t[first..last) as a group of their own (segment space from 0,
+// global-scale slots of the workspace from amax_slot).
+GroupParams subgroup(const GroupParams& p, int first, int last, int amax_slot) {
+    GroupParams q = p;
+    q.count = last - first;
+    int64_t seg = 0;
+    for (int k = 0; k < q.count; k++) {
+        q.t[k] = p.t[first + k];
+        q.t[k].seg_begin = seg;
+        seg += (q.t[k].nseg + kGroupCtaSegments - 1) / kGroupCtaSegments * kGroupCtaSegments;
+    }
+    q.total_seg = seg;
+    q.amax_bits = p.amax_bits + amax_slot;
+    return q;
+}
+
+// Pipelined schedule of in-launch global scales (p.count >= 2).  The last
+// tensor of p (the largest: p is in ascending size) goes first:
+//   reduce(last)  full GPU, ordinary launch;
+//   sweep(last)   waits for it, then lets the next grid be scheduled; at most
+//                 kPipeSweepCtas CTAs per SM when the rest is over half its size;
+//   reduce(rest)  co-resident with sweep(last) on the registers the sweep
+//                 leaves free (32 per thread), completes after it;
+//   sweep(rest)   one grouped sweep of the other tensors, waits for reduce(rest).
+// The three later grids are programmatic dependent launches, so no CTA waits
+// on a flag and each grid waits only for the one launched just before it.
+// Only the first tensor's reduction stays exposed: the others overlap a sweep
+// bound by the FP32 pipe, not by HBM.
 template <int DT, int METHOD, int OBJ, int BLOCK>
-cudaError_t launch_dyn_or_static(const GroupParams& p, int sms, cudaStream_t s) {
-    return p.dyn ? launch_group<DT, METHOD, OBJ, BLOCK, 1>(p, sms, s) : launch_group<DT, METHOD, OBJ, BLOCK, 0>(p, sms, s);
+cudaError_t launch_group_pipelined(const GroupParams& p, int sms, cudaStream_t s) {
+    const GroupParams a = subgroup(p, p.count - 1, p.count, 0);
+    const GroupParams b = subgroup(p, 0, p.count - 1, 1);
+    unsigned* ticket = p.arrived;
+    cudaError_t e = cudaMemsetAsync(p.amax_bits, 0, kGroupWorkspace, s);
+    if (e != cudaSuccess) return e;
+    group_reduce_kernel<DT><<<(unsigned)sms * (2048 / kReduceThreads), kReduceThreads, 0, s>>>(a, ticket);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    int occ = 1;
+    const bool big_rest = b.total_seg > a.total_seg / 2;
+    const int64_t grid_a = sweep_grid<DT, METHOD, OBJ, BLOCK, 2>(a, sms, &occ, big_rest ? kPipeSweepCtas : 0);
+    e = launch_dependent(quantize_group_kernel<DT, METHOD, OBJ, BLOCK, 2>, grid_a, kSweepThreads, s, a);
+    if (e != cudaSuccess) return e;
+    // reduction CTAs that fit beside `occ` sweep CTAs per SM: each of its warps
+    // takes 32 x 32 registers on one of the four schedulers' 16K-register files
+    static std::atomic<int> regs_cache[kOccDevices];
+    int dev = -1, regs = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < kOccDevices)
+        regs = regs_cache[dev].load(std::memory_order_relaxed);
+    if (regs <= 0) {
+        cudaFuncAttributes fa;
+        e = cudaFuncGetAttributes(&fa, quantize_group_kernel<DT, METHOD, OBJ, BLOCK, 2>);
+        if (e != cudaSuccess) return e;
+        regs = fa.numRegs;
+        if (dev >= 0 && dev < kOccDevices) regs_cache[dev].store(regs, std::memory_order_relaxed);
+    }
+    const int warp_regs = (regs + 7) / 8 * 8 * 32;
+    const int sweep_warps_per_sched = (occ * (kSweepThreads / 32) + 3) / 4;
+    const int free_per_sched = 16384 - sweep_warps_per_sched * warp_regs;
+    int per_sm = free_per_sched / (32 * 32) / (kReduceThreads / 32 / 4);
+    per_sm = per_sm < 1 ? 1 : (per_sm > 2048 / kReduceThreads ? 2048 / kReduceThreads : per_sm);
+    e = launch_dependent(group_reduce_kernel<DT>, (int64_t)sms * per_sm, kReduceThreads, s, b, ticket + 1);
+    if (e != cudaSuccess) return e;
+    const int64_t grid_b = sweep_grid<DT, METHOD, OBJ, BLOCK, 2>(b, sms, nullptr);
+    return launch_dependent(quantize_group_kernel<DT, METHOD, OBJ, BLOCK, 2>, grid_b, kSweepThreads, s, b);
+}
+
+template <int DT, int METHOD, int OBJ, int BLOCK>
+cudaError_t launch_schedule(const GroupParams& p, int sms, cudaStream_t s) {
+    if (!p.dyn) return launch_group<DT, METHOD, OBJ, BLOCK, 0>(p, sms, s);
+    if (p.pipelined && METHOD == 0 && p.count >= 2) return launch_group_pipelined<DT, METHOD, OBJ, BLOCK>(p, sms, s);
+    return launch_group<DT, METHOD, OBJ, BLOCK, 1>(p, sms, s);
 }
 
 template <int DT, int METHOD, int OBJ>
 cudaError_t launch_block(const GroupParams& p, int block, int sms, cudaStream_t s) {
     switch (block) {
-        case 16: return launch_dyn_or_static<DT, METHOD, OBJ, 16>(p, sms, s);
-        case 32: return launch_dyn_or_static<DT, METHOD, OBJ, 32>(p, sms, s);
-        default: return launch_dyn_or_static<DT, METHOD, OBJ, 64>(p, sms, s);
+        case 16: return launch_schedule<DT, METHOD, OBJ, 16>(p, sms, s);
+        case 32: return launch_schedule<DT, METHOD, OBJ, 32>(p, sms, s);
+        default: return launch_schedule<DT, METHOD, OBJ, 64>(p, sms, s);
     }
 }
 

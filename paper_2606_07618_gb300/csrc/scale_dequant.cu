@@ -16,15 +16,6 @@
 
 namespace nvfp4 {
 
-// Programmatic dependent launch: the running grid lets a kernel launched after
-// it with cudaLaunchAttributeProgrammaticStreamSerialization be scheduled early;
-// that kernel's griddepcontrol.wait returns once this grid has completed and
-// its writes are visible (and at once when it was launched the ordinary way).
-__device__ __forceinline__ void grid_launch_dependents() {
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-
 __device__ __forceinline__ void amax_acc(float v, float& m, int& bad) {
     if (!isfinite(v)) bad = 1;
     m = fmaxf(m, fabsf(v));                  // fmaxf drops NaN, keeps inf

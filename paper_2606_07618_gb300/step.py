@@ -62,8 +62,15 @@ class QuantizeStep:
     def numel(self) -> int:
         return sum(x.numel() for x in self.xs)
 
+    @property
+    def pipelined(self) -> bool:
+        """Whether the grouped call takes the pipelined schedule (the library's
+        choice: a ScaleSweep over at least two tensors and 2^25 elements)."""
+        return not self.fused and len(self.xs) >= 2 and self.numel >= 1 << 25
+
     def __call__(self, stream=None):
-        """ScaleSweep over every tensor (one launch, plus a workspace memset)."""
+        """ScaleSweep over every tensor (one library call: a workspace memset,
+        then one cooperative launch or the pipelined schedule's four)."""
         if self.fused:
             o = self.outs[0]
             win = (B.NVFP4_WINDOW_DEFAULT, B.NVFP4_WINDOW_DEFAULT)

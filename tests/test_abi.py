@@ -31,7 +31,7 @@ def test_header_declares_the_api():
         "nvfp4_dynamic_workspace", "scalesweep_quantize_dynamic", "absmax_quantize_dynamic",
         "nvfp4_optimal_scale", "nvfp4_ldlq_prepare_workspace", "nvfp4_ldlq_prepare", "nvfp4_ldlq_workspace",
         "ldlq_quantize", "scalesweep_quantize_group_workspace", "scalesweep_quantize_group",
-        "absmax_quantize_group", "nvfp4_selftest_wait_timeout", "nvfp4_row_shard_layout"])
+        "scalesweep_quantize_group_scheduled", "absmax_quantize_group", "nvfp4_selftest_wait_timeout", "nvfp4_row_shard_layout"])
 
 
 def test_library_exports_every_declared_symbol(L):
@@ -168,6 +168,12 @@ def test_group_validation_without_gpu(L):
     assert g(desc(), block=8) == 2                    # block not in {16, 32, 64}
     assert g(desc({"cols": 48}), block=32) == 1       # cols % block
     assert g(desc({"sf_swizzled": FAKE + 0x5000000}), block=32) == 2   # swizzled scales need block 16
+    sch = lambda d, schedule, n=2: L.scalesweep_quantize_group_scheduled(d, n, 0, 16, 0, f(256.0), S, st, ws, 256,
+                                                                          schedule, None)
+    assert sch(desc(), 3) == 1                        # unknown schedule
+    assert sch(desc(), -1) == 1
+    assert sch(desc(), 2, n=0) == 1                   # the other checks apply under every schedule
+    assert sch(desc({"x": FAKE + 2}), 2) == 3
     assert a(desc(), n=0) == 1
     assert a(desc(), block=128) == 2
     assert a(desc(), ws=None) == 1
@@ -208,6 +214,8 @@ int main(void) {
     printf("NVFP4_SF_LINEAR %d\nNVFP4_SF_SWIZZLED %d\n", NVFP4_SF_LINEAR, NVFP4_SF_SWIZZLED);
     printf("NVFP4_WINDOW_DEFAULT %d\nNVFP4_WINDOW_TIGHT %d\nNVFP4_GROUP_MAX %d\n", NVFP4_WINDOW_DEFAULT,
            NVFP4_WINDOW_TIGHT, NVFP4_GROUP_MAX);
+    printf("NVFP4_GROUP_SCHEDULE_AUTO %d\nNVFP4_GROUP_SCHEDULE_TWO_PHASE %d\nNVFP4_GROUP_SCHEDULE_PIPELINED %d\n",
+           NVFP4_GROUP_SCHEDULE_AUTO, NVFP4_GROUP_SCHEDULE_TWO_PHASE, NVFP4_GROUP_SCHEDULE_PIPELINED);
     return 0;
 }
 ''')
@@ -224,7 +232,8 @@ int main(void) {
         f = getattr(B.RowShard, name)
         assert vals["shard_" + name] == [f.offset, f.size], name
     for name in ("NVFP4_IN_BF16", "NVFP4_IN_F32", "NVFP4_OBJ_MSE", "NVFP4_OBJ_WMSE", "NVFP4_SF_LINEAR",
-                 "NVFP4_SF_SWIZZLED", "NVFP4_WINDOW_DEFAULT", "NVFP4_WINDOW_TIGHT", "NVFP4_GROUP_MAX"):
+                 "NVFP4_SF_SWIZZLED", "NVFP4_WINDOW_DEFAULT", "NVFP4_WINDOW_TIGHT", "NVFP4_GROUP_MAX",
+                 "NVFP4_GROUP_SCHEDULE_AUTO", "NVFP4_GROUP_SCHEDULE_TWO_PHASE", "NVFP4_GROUP_SCHEDULE_PIPELINED"):
         assert vals[name] == [getattr(B, name)], name
 
 
@@ -251,7 +260,7 @@ def _ctype_of(param):
     t = decl.replace("const", "").strip()
     return {"int": ctypes.c_int, "int64_t": ctypes.c_int64, "float": ctypes.c_float, "size_t": ctypes.c_size_t,
             "nvfp4_dtype": ctypes.c_int, "nvfp4_objective": ctypes.c_int, "nvfp4_sf_layout": ctypes.c_int,
-            "nvfp4_status": ctypes.c_int}[t]
+            "nvfp4_group_schedule": ctypes.c_int, "nvfp4_status": ctypes.c_int}[t]
 
 
 def _declared_return_types():

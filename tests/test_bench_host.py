@@ -89,7 +89,7 @@ def test_traffic_record_is_dropped_when_sources_change(tmp_path, monkeypatch):
 
 
 def test_committed_traffic_records_are_well_formed():
-    for name in ("quantize_group_kernel_qwen72b_traffic.json",):
+    for name in ("quantize_group_pipelined_qwen72b_traffic.json",):
         with open(os.path.join(bench.ROOT, "profiles", name)) as f:
             rec = json.load(f)
         assert rec["source_files"] and len(rec["source_sha256"]) == 64
@@ -98,6 +98,23 @@ def test_committed_traffic_records_are_well_formed():
         assert 1.0 < rec["dram_bytes_per_element"] < 6.0
         for fn in rec["source_files"]:
             assert os.path.exists(os.path.join(bench.ROOT, fn)), fn
+        if "per_launch" in rec:                # the step's launches add up to the totals
+            rd = sum(x["bytes"] for x in rec["per_launch"] if x["metric"] == "dram__bytes_read.sum")
+            wr = sum(x["bytes"] for x in rec["per_launch"] if x["metric"] == "dram__bytes_write.sum")
+            assert (rd, wr) == (rec["dram_read_bytes"], rec["dram_write_bytes"])
+
+
+def test_step_schedule_threshold_matches_the_library():
+    """QuantizeStep.pipelined describes the library's automatic choice; its
+    element threshold is the one the library's grouped launch uses."""
+    import re
+    from paper_2606_07618_gb300 import step as ST
+    src = open(os.path.join(bench.ROOT, "paper_2606_07618_gb300", "csrc", "group_kernels.h")).read()
+    m = re.search(r"kPipelineMinElements\s*=\s*int64_t\(1\)\s*<<\s*(\d+);", src)
+    assert m is not None
+    shift = int(m.group(1))
+    step_src = open(ST.__file__).read()
+    assert f"self.numel >= 1 << {shift}" in step_src
 
 
 def test_workload_roofline_terms():

@@ -64,7 +64,8 @@ def make_group(dtype, obj, seed=0, shapes=SHAPES, row_weights=(3,)):
     return xs, ws, strides
 
 
-def run_group(B, xs, ws, strides, obj, D=256.0, S_in=None, ws_buf=None, status=None, block=16, method=0):
+def run_group(B, xs, ws, strides, obj, D=256.0, S_in=None, ws_buf=None, status=None, block=16, method=0,
+              schedule=None):
     dev_x = [x.to(DEV) for x in xs]
     dev_w = [w.to(DEV) if w is not None else None for w in ws]
     outs = [B.empty_outputs(x.shape[0], x.shape[1], block, device=DEV, linear=True, swizzled=block == 16)
@@ -77,7 +78,8 @@ def run_group(B, xs, ws, strides, obj, D=256.0, S_in=None, ws_buf=None, status=N
                                [o["sf_swizzled"] for o in outs])
     dt = B.NVFP4_IN_BF16 if xs[0].dtype == torch.bfloat16 else B.NVFP4_IN_F32
     st = status if status is not None else torch.zeros(1, dtype=torch.int32, device=DEV)
-    call = (lambda d, S_, ws_: B.scalesweep_quantize_group(desc, dt, obj, d, S_, st, ws_, block=block)) \
+    call = (lambda d, S_, ws_: B.scalesweep_quantize_group(desc, dt, obj, d, S_, st, ws_, block=block,
+                                                           schedule=schedule)) \
         if method == 0 else (lambda d, S_, ws_: B.absmax_quantize_group(desc, dt, d, S_, st, ws_, block=block))
     if S_in is None:
         S = torch.full((len(xs),), -1.0, device=DEV)
@@ -121,11 +123,15 @@ def check_against_per_tensor(B, xs, ws, strides, obj, S, outs, dev_x, dev_w, sta
                 assert torch.equal(outs[i][k], o1[k]), f"tensor {i}: {k}"
 
 
+SCHEDULES = [None, 1, 2]        # the library's choice, two-phase, pipelined
+
+
+@pytest.mark.parametrize("schedule", SCHEDULES)
 @pytest.mark.parametrize("obj", [0, 1])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
-def test_group_dynamic_matches_oracle_and_per_tensor(B, dtype, obj):
+def test_group_dynamic_matches_oracle_and_per_tensor(B, dtype, obj, schedule):
     xs, ws, strides = make_group(dtype, obj, seed=1)
-    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, obj)
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, obj, schedule=schedule)
     assert st.item() == 0
     check_against_per_tensor(B, xs, ws, strides, obj, S, outs, dev_x, dev_w)
     for i, x in enumerate(xs):
@@ -142,20 +148,24 @@ def test_group_dynamic_matches_oracle_and_per_tensor(B, dtype, obj):
 SHAPES64 = [(130, 192), (1, 64), (37, 128), (300, 512), (0, 64), (1000, 1024), (64, 320)]
 
 
-@pytest.mark.parametrize("dyn", [True, False])
+@pytest.mark.parametrize("dyn", [True, False, "pipelined"])
 @pytest.mark.parametrize("block,obj,method", [(32, 0, 0), (32, 1, 0), (64, 0, 0), (64, 1, 0),
                                               (16, 0, 1), (32, 0, 1), (64, 0, 1)])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
 def test_group_blocks_and_absmax(B, dtype, block, obj, method, dyn):
     """Blocks of 32 and 64 (two and four lanes per block) and the grouped AbsMax
     launch: every tensor equals the oracle (near-tie rule) and, bit for bit,
-    the per-tensor call with the same scale."""
+    the per-tensor call with the same scale.  "pipelined": dynamic scales under
+    the pipelined schedule (AbsMax has no such schedule)."""
+    if dyn == "pipelined" and method == 1:
+        pytest.skip("the pipelined schedule is a ScaleSweep schedule")
     xs, ws, strides = make_group(dtype, obj, seed=7 + block + 3 * method, shapes=SHAPES64)
     S_in = None
     if not dyn:
         S_in = torch.tensor([oracle.global_scale(x.float().numpy(), 256.0)[0] if x.numel() else 1.0 for x in xs],
                             dtype=torch.float32, device=DEV)
-    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, obj, S_in=S_in, block=block, method=method)
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, obj, S_in=S_in, block=block, method=method,
+                                          schedule=2 if dyn == "pipelined" else None)
     assert st.item() == 0
     check_against_per_tensor(B, xs, ws, strides, obj, S, outs, dev_x, dev_w, static=not dyn, block=block,
                              method=method)
@@ -183,16 +193,37 @@ def test_group_static_scales(B, obj):
     check_against_per_tensor(B, xs, ws, strides, obj, S, outs, dev_x, dev_w, static=True)
 
 
-def test_group_single_tensor_and_many_tensors(B):
+@pytest.mark.parametrize("schedule", SCHEDULES)
+def test_group_single_tensor_and_many_tensors(B, schedule):
     # one tensor; and the maximum of 16 tensors of assorted small shapes
     xs, ws, strides = make_group(torch.bfloat16, 1, seed=3, shapes=[(513, 4096)], row_weights=())
-    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, 1)
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, 1, schedule=schedule)
     check_against_per_tensor(B, xs, ws, strides, 1, S, outs, dev_x, dev_w)
     shapes = [(1 + 37 * i, 16 * (1 + (5 * i) % 23)) for i in range(16)]
     xs, ws, strides = make_group(torch.bfloat16, 0, seed=4, shapes=shapes)
-    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, 0)
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, 0, schedule=schedule)
     assert st.item() == 0
     check_against_per_tensor(B, xs, ws, strides, 0, S, outs, dev_x, dev_w)
+
+
+@pytest.mark.parametrize("obj", [0, 1])
+def test_group_schedules_agree_on_large_tensors(B, obj):
+    """Tensors large enough that the pipelined schedule's reduction of the
+    smaller ones runs beside the largest one's sweep (bf16, 117M elements in
+    three tensors): S, codes and both scale layouts are the same bytes under
+    both schedules."""
+    shapes = [(4096, 4096), (1024, 8192), (12288, 8192)]
+    xs = [W.small_tensor(r, c, 60 + i, dist="normal", std=0.02, outliers=4, mult=20.0) for i, (r, c) in
+          enumerate(shapes)]
+    ws = [torch.exp(torch.randn(c, generator=torch.Generator().manual_seed(70 + i))) if obj else None
+          for i, (_, c) in enumerate(shapes)]
+    res = [run_group(B, xs, ws, [0] * 3, obj, schedule=sch) for sch in (1, 2)]
+    (S1, st1, o1, _, _), (S2, st2, o2, _, _) = res
+    assert st1.item() == 0 and st2.item() == 0 and torch.equal(S1, S2)
+    for i, (xn, Si) in enumerate(zip(xs, S1.tolist())):
+        assert Si == np.float32(oracle.global_scale(xn.float().numpy(), 256.0)[0])
+        for k in ("codes", "sf_linear", "sf_swizzled"):
+            assert torch.equal(o1[i][k], o2[i][k]), (i, k)
 
 
 def test_group_llama_layer_full_size(B):
@@ -216,12 +247,13 @@ def test_group_llama_layer_full_size(B):
         compare_quantize(xs_np[idx], So, 16, 1, ws[i], 0, sub, ref)
 
 
-def test_group_nonfinite_flag_reuse_and_empty(B):
+@pytest.mark.parametrize("schedule", SCHEDULES)
+def test_group_nonfinite_flag_reuse_and_empty(B, schedule):
     xs, ws, strides = make_group(torch.bfloat16, 0, seed=5)
     wsb = torch.empty(B.scalesweep_quantize_group_workspace(), dtype=torch.uint8, device=DEV)
     ref = None
     for _ in range(3):                                             # one workspace, back to back
-        S, st, outs, _, _ = run_group(B, xs, ws, strides, 0, ws_buf=wsb)
+        S, st, outs, _, _ = run_group(B, xs, ws, strides, 0, ws_buf=wsb, schedule=schedule)
         assert st.item() == 0
         if ref is None:
             ref = (S.clone(), outs)
@@ -232,15 +264,15 @@ def test_group_nonfinite_flag_reuse_and_empty(B):
                     assert torch.equal(a[k], b[k])
     bad = [x.clone() for x in xs]
     bad[3][5, 7] = float("inf")
-    S, st, _, _, _ = run_group(B, bad, ws, strides, 0, ws_buf=wsb)
-    assert st.item() & 1
+    S, st, _, _, _ = run_group(B, bad, ws, strides, 0, ws_buf=wsb, schedule=schedule)
+    assert st.item() == 1
     assert S[3].item() == float("inf") and torch.equal(S[:3], ref[0][:3])
     bad = [x.clone() for x in xs]
     bad[5][0, 0] = float("nan")
-    S, st, _, _, _ = run_group(B, bad, ws, strides, 0, ws_buf=wsb)
-    assert st.item() & 1 and S[5].item() == ref[0][5].item()         # NaN is skipped by the max
+    S, st, _, _, _ = run_group(B, bad, ws, strides, 0, ws_buf=wsb, schedule=schedule)
+    assert st.item() == 1 and S[5].item() == ref[0][5].item()        # NaN is skipped by the max
     empty = [torch.empty(0, 64, dtype=torch.bfloat16), torch.empty(3, 0, dtype=torch.bfloat16)]
-    S, st, _, _, _ = run_group(B, empty, [None, None], [0, 0], 0, ws_buf=wsb)
+    S, st, _, _, _ = run_group(B, empty, [None, None], [0, 0], 0, ws_buf=wsb, schedule=schedule)
     assert S.tolist() == [0.0, 0.0] and st.item() == 0
 
 
@@ -301,12 +333,14 @@ def test_group_output_guard_bytes_untouched(B):
         assert torch.equal(sfs[i], o1["sf_swizzled"])
 
 
-def test_group_dynamic_in_cuda_graph(B):
-    """The grouped call (workspace memset + cooperative launch) captured in a
-    CUDA graph and replayed gives the eager results; the library neither
-    allocates nor synchronises, so it can be captured."""
+@pytest.mark.parametrize("schedule", [1, 2])
+def test_group_dynamic_in_cuda_graph(B, schedule):
+    """The grouped call (workspace memset, then the cooperative launch or the
+    pipelined schedule's four launches) captured in a CUDA graph and replayed
+    gives the eager results; the library neither allocates nor synchronises,
+    so it can be captured."""
     xs, ws, strides = make_group(torch.bfloat16, 1, seed=8, shapes=[(300, 512), (64, 80), (1024, 256)])
-    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, 1)
+    S, st, outs, dev_x, dev_w = run_group(B, xs, ws, strides, 1, schedule=3 - schedule)
     outs2 = [B.empty_outputs(x.shape[0], x.shape[1], 16, device=DEV, linear=True, swizzled=True) for x in xs]
     desc = B.group_descriptors(dev_x, dev_w, strides, [o["codes"] for o in outs2], [o["sf_linear"] for o in outs2],
                                [o["sf_swizzled"] for o in outs2])
@@ -316,10 +350,11 @@ def test_group_dynamic_in_cuda_graph(B):
     g = torch.cuda.CUDAGraph()
     s = torch.cuda.Stream()
     with torch.cuda.stream(s):
-        B.scalesweep_quantize_group(desc, B.NVFP4_IN_BF16, 1, 256.0, S2, st2, wsb, stream=s)   # warm-up
+        B.scalesweep_quantize_group(desc, B.NVFP4_IN_BF16, 1, 256.0, S2, st2, wsb, stream=s,
+                                    schedule=schedule)                                         # warm-up
     torch.cuda.synchronize()
     with torch.cuda.graph(g, stream=s):
-        B.scalesweep_quantize_group(desc, B.NVFP4_IN_BF16, 1, 256.0, S2, st2, wsb, stream=s)
+        B.scalesweep_quantize_group(desc, B.NVFP4_IN_BF16, 1, 256.0, S2, st2, wsb, stream=s, schedule=schedule)
     for _ in range(2):
         for o in outs2:
             o["codes"].zero_()
