@@ -238,7 +238,6 @@ __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand*
                                                bool valid, u64 E2, bool usable, u64 (&w2)[8], const float*& wkey) {
     constexpr int SEGS = BLOCK / 16;
     constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
-    constexpr int FIX_K = 7 - FIX_LO + 1;
     u64 y2[8];
     float m = 0.0f;
     if (valid) {
@@ -277,20 +276,10 @@ __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand*
     const bool zero = zero_block(usable, m);
     int bestc;
     if (METHOD == 0) {
-        float best = __int_as_float(0x7f800000);
+        float best;
         const int I0 = e4m3_floor_code(__fdiv_rn(m, 6.0f));
         const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
-        int bk = 0;
-#pragma unroll
-        for (int k = 0; k < FIX_K; k++) {
-            const Cand cd = tb[k];
-            const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));
-            if (L < best) {
-                best = L;
-                bk = k;
-            }
-        }
-        bestc = I0 + FIX_LO + bk;
+        bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK>(y2, w2, m, tb, best);
     } else {
         bestc = max((int)e4m3_rn_code(__fdiv_rn(m, 6.0f)), 1);
     }

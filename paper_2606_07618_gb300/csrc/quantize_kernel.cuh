@@ -178,6 +178,63 @@ __device__ __forceinline__ float group_max(float v) {
     return v;
 }
 
+// Default-window argmin (FIX windows: [I0-3, I0+7] for MSE with blocks of
+// 16, [I0-8, I0+7] otherwise) over the candidate table entries tb[0..FIX_K),
+// tb[k] being code I0 + FIX_LO + k.  Returns the offset k of the lowest code
+// whose loss is minimal and sets `best` to that loss.
+//
+// MSE: the lowest NB offsets are visited last, in descending order, and a warp
+// skips one when, for every lane, the block's largest element alone already
+// costs more than the lane's best loss so far.  That single term, fl(e_m^2)
+// with e_m = cand_err1(m, ...), is the term the candidate's loss accumulates
+// for that element (fma(e, e, acc) over non-negative terms, then sums of
+// non-negative partial losses), and rounding is monotone, so the loss is at
+// least the term: a skipped candidate has a loss above the final best and can
+// neither win nor tie.  The losses that are computed are the same values in
+// the same order, with ties going to the lowest code (<= for the codes below
+// every code already visited), so the result is the full sweep's, bit for
+// bit.  On the low offsets the block's largest element saturates (6 v_c < m),
+// which makes the bound tight: on the synthetic Qwen2.5-72B-shaped weights a
+// warp skips offset 0 of the 11 MSE candidates (I0-3) in 96% of its visits and
+// ~5 of the 16 candidates of blocks of 32/64.  WMSE has no cheap bound of this
+// kind (the largest element's weight would first have to be found), so NB = 0.
+template <int OBJ, int BLOCK>
+__host__ __device__ constexpr int bound_offsets() {
+    return OBJ != 0 ? 0 : (BLOCK == 16 ? 1 : (BLOCK == 32 ? 5 : 4));
+}
+
+template <int OBJ, int BLOCK>
+__device__ __forceinline__ int default_window_argmin(const u64 (&y2)[8], const u64 (&w2)[8], float m, const Cand* tb,
+                                                     float& best) {
+    constexpr int SEGS = BLOCK / 16;
+    constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
+    constexpr int FIX_K = 7 - FIX_LO + 1;
+    constexpr int NB = bound_offsets<OBJ, BLOCK>();
+    best = __int_as_float(0x7f800000);
+    int bk = 0;
+#pragma unroll
+    for (int k = NB; k < FIX_K; k++) {
+        const Cand cd = tb[k];
+        const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));
+        if (L < best) {
+            best = L;
+            bk = k;
+        }
+    }
+#pragma unroll
+    for (int k = NB - 1; k >= 0; k--) {
+        const Cand cd = tb[k];
+        const float e = cand_err1(m, cd.r, (uint16_t)cd.nv);
+        if (__all_sync(0xffffffffu, __fmul_rn(e, e) > best)) continue;       // warp-uniform
+        const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));
+        if (L <= best) {
+            best = L;
+            bk = k;
+        }
+    }
+    return bk;
+}
+
 // n / d for 32-bit n by multiply-high and shifts (Granlund-Montgomery).
 __device__ __forceinline__ uint32_t fast_div(uint32_t n, const FastDiv& d) {
     const uint32_t t = __umulhi(n, d.mul);
@@ -187,10 +244,6 @@ __device__ __forceinline__ uint32_t fast_div(uint32_t n, const FastDiv& d) {
 #ifndef NVFP4_QMINB
 #define NVFP4_QMINB 1
 #endif
-#ifndef NVFP4_CAND_UNROLL
-#define NVFP4_CAND_UNROLL 16
-#endif
-constexpr int kCandUnroll = NVFP4_CAND_UNROLL;
 
 // Dynamic (per-call) global scale inside the sweep launch: every CTA folds the
 // max |x| of its grid-stride share into one partial, all CTAs meet at a grid
@@ -327,7 +380,6 @@ template <int DT, int METHOD, int OBJ, int BLOCK, int FIX, int DYN>
 __global__ void __launch_bounds__(256, quantize_min_blocks<METHOD, DT>()) quantize_kernel(QuantParams p) {
     constexpr int SEGS = BLOCK / 16;
     constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
-    constexpr int FIX_K = 7 - FIX_LO + 1;
     __shared__ Cand tab[kTabN];
     build_table(tab);
     __syncthreads();
@@ -407,17 +459,7 @@ __global__ void __launch_bounds__(256, quantize_min_blocks<METHOD, DT>()) quanti
             const int I0 = e4m3_floor_code(sbase);
             if (FIX) {
                 const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
-                int bk = 0;
-#pragma unroll kCandUnroll
-                for (int k = 0; k < FIX_K; k++) {
-                    const Cand cd = tb[k];
-                    const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));
-                    if (L < best) {
-                        best = L;
-                        bk = k;
-                    }
-                }
-                bestc = I0 + FIX_LO + bk;
+                bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK>(y2, w2, m, tb, best);
             } else {
                 int lo_off = p.win_lo;
                 if ((p.tight & 2) && I0 >= 16 && I0 <= 120) {
