@@ -235,7 +235,8 @@ __global__ void __launch_bounds__(kReduceThreads, 2048 / kReduceThreads)
 // are loaded once per tensor.
 template <int DT, int METHOD, int OBJ, int BLOCK>
 __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand* tab, const Raw& cur, int64_t g,
-                                               bool valid, u64 E2, bool usable, u64 (&w2)[8], const float*& wkey) {
+                                               bool valid, u64 E2, bool usable, u64 (&w2)[8], const float*& wkey,
+                                               bool& wok) {
     constexpr int SEGS = BLOCK / 16;
     constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
     u64 y2[8];
@@ -271,6 +272,7 @@ __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand*
                 w2[2 * j + 1] = pack2(__uint_as_float(a.z), __uint_as_float(a.w));
             }
             wkey = wp;
+            wok = weights_nonneg(w2);
         }
     }
     const bool zero = zero_block(usable, m);
@@ -279,7 +281,7 @@ __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand*
         float best;
         const int I0 = e4m3_floor_code(__fdiv_rn(m, 6.0f));
         const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
-        bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK>(y2, w2, m, tb, best);
+        bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK>(y2, w2, m, tb, best, wok);
     } else {
         bestc = max((int)e4m3_rn_code(__fdiv_rn(m, 6.0f)), 1);
     }
@@ -379,6 +381,7 @@ __global__ void __launch_bounds__(kSweepThreads, group_min_blocks<METHOD, OBJ>()
 #pragma unroll
     for (int j = 0; j < 8; j++) w2[j] = 0ull;
     const float* wkey = nullptr;
+    bool wok = true;                                     // the lane's weights are all >= 0
     Raw cur;
     if (cbase < total) {
         const int64_t g = cbase + tid - p.t[t].seg_begin;
@@ -410,7 +413,7 @@ __global__ void __launch_bounds__(kSweepThreads, group_min_blocks<METHOD, OBJ>()
                 const int64_t gn = nb + tid - p.t[tn].seg_begin;
                 if (gn < p.t[tn].nseg) load_raw<DT>(p.t[tn].x, gn, nxt);
             }
-            sweep_segments<DT, METHOD, OBJ, BLOCK>(d, tab, cur, g, valid, E2, usable, w2, wkey);
+            sweep_segments<DT, METHOD, OBJ, BLOCK>(d, tab, cur, g, valid, E2, usable, w2, wkey, wok);
             cur = nxt;
         }
         t = tensor_at(p, t, cbase);

@@ -183,29 +183,35 @@ __device__ __forceinline__ float group_max(float v) {
 // tb[k] being code I0 + FIX_LO + k.  Returns the offset k of the lowest code
 // whose loss is minimal and sets `best` to that loss.
 //
-// MSE: the lowest NB offsets are visited last, in descending order, and a warp
+// The lowest NB offsets are visited last, in descending order, and a warp
 // skips one when, for every lane, the block's largest element alone already
-// costs more than the lane's best loss so far.  That single term, fl(e_m^2)
-// with e_m = cand_err1(m, ...), is the term the candidate's loss accumulates
-// for that element (fma(e, e, acc) over non-negative terms, then sums of
-// non-negative partial losses), and rounding is monotone, so the loss is at
-// least the term: a skipped candidate has a loss above the final best and can
-// neither win nor tie.  The losses that are computed are the same values in
-// the same order, with ties going to the lowest code (<= for the codes below
-// every code already visited), so the result is the full sweep's, bit for
-// bit.  On the low offsets the block's largest element saturates (6 v_c < m),
-// which makes the bound tight: on the synthetic Qwen2.5-72B-shaped weights a
-// warp skips offset 0 of the 11 MSE candidates (I0-3) in 96% of its visits and
-// ~5 of the 16 candidates of blocks of 32/64.  WMSE has no cheap bound of this
-// kind (the largest element's weight would first have to be found), so NB = 0.
+// costs more than the lane's best loss so far.  That single term -- fl(e_m^2)
+// for MSE, fl(fl(w_m e_m) e_m) for WMSE, with e_m = cand_err1(m, ...) and w_m
+// the weight of an element whose |y| is m -- is the term the candidate's loss
+// accumulates for that element, every other term is non-negative (squares;
+// WMSE: only while the lane's weights are non-negative, `wok`, else no skip),
+// and rounding is monotone, so the loss is at least the term: a skipped
+// candidate has a loss above the final best and can neither win nor tie.  The
+// losses that are computed are the same values in the same order, with ties
+// going to the lowest code (<= for the codes below every code already
+// visited), so the result is the full sweep's, bit for bit.  On the low
+// offsets the block's largest element saturates (6 v_c < m), which makes the
+// bound tight: on the synthetic Qwen2.5-72B-shaped weights a warp skips offset
+// 0 of the 11 MSE candidates (I0-3) in 96% of its visits, ~5 of the 16 MSE
+// candidates of blocks of 32/64, and ~2.4 of the 16 WMSE candidates of blocks
+// of 16.  NB per objective and block as measured on those weights (grouped
+// call, ms; every NB gave the same output bytes): WMSE block 16, NB 0/2/3/4/5:
+// 1.409/1.369/1.336/1.325/1.334 with static scales; WMSE blocks of 32 and 64
+// gain nothing (a single element's term is small against a 32- or 64-element
+// loss) and lose up to 2% at NB 4, so they keep the plain sweep.
 template <int OBJ, int BLOCK>
 __host__ __device__ constexpr int bound_offsets() {
-    return OBJ != 0 ? 0 : (BLOCK == 16 ? 1 : (BLOCK == 32 ? 5 : 4));
+    return OBJ != 0 ? (BLOCK == 16 ? 4 : 0) : (BLOCK == 16 ? 1 : (BLOCK == 32 ? 5 : 4));
 }
 
 template <int OBJ, int BLOCK>
 __device__ __forceinline__ int default_window_argmin(const u64 (&y2)[8], const u64 (&w2)[8], float m, const Cand* tb,
-                                                     float& best) {
+                                                     float& best, bool wok = true) {
     constexpr int SEGS = BLOCK / 16;
     constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
     constexpr int FIX_K = 7 - FIX_LO + 1;
@@ -221,11 +227,29 @@ __device__ __forceinline__ int default_window_argmin(const u64 (&y2)[8], const u
             bk = k;
         }
     }
+    if (NB == 0) return bk;
+    float wm = 1.0f;
+    if (OBJ == 1) {
+        // weight of an element of this lane whose |y| is the block max (0 if
+        // none), then the largest over the block's lanes: every element at the
+        // max has the same error, so any of their weights gives a valid term
+        wm = 0.0f;
+#pragma unroll
+        for (int j = 0; j < 8; j++) {
+            float a, b, wa, wb;
+            unpack2(y2[j], a, b);
+            unpack2(w2[j], wa, wb);
+            wm = fabsf(a) == m ? wa : wm;
+            wm = fabsf(b) == m ? wb : wm;
+        }
+        wm = group_max<SEGS>(wok ? wm : __int_as_float(0x7fc00000));   // negative or NaN weights: no skip
+    }
 #pragma unroll
     for (int k = NB - 1; k >= 0; k--) {
         const Cand cd = tb[k];
         const float e = cand_err1(m, cd.r, (uint16_t)cd.nv);
-        if (__all_sync(0xffffffffu, __fmul_rn(e, e) > best)) continue;       // warp-uniform
+        const float term = OBJ == 1 ? __fmul_rn(__fmul_rn(wm, e), e) : __fmul_rn(e, e);
+        if (__all_sync(0xffffffffu, term > best)) continue;                  // warp-uniform
         const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));
         if (L <= best) {
             best = L;
@@ -233,6 +257,18 @@ __device__ __forceinline__ int default_window_argmin(const u64 (&y2)[8], const u
         }
     }
     return bk;
+}
+
+// Whether all 16 weights of a segment are non-negative (NaN counts as not).
+__device__ __forceinline__ bool weights_nonneg(const u64 (&w2)[8]) {
+    float lo = __int_as_float(0x7f800000);
+#pragma unroll
+    for (int j = 0; j < 8; j++) {
+        float a, b;
+        unpack2(w2[j], a, b);
+        asm("min.NaN.f32 %0, %1, %2, %3;" : "=f"(lo) : "f"(lo), "f"(a), "f"(b));
+    }
+    return lo >= 0.0f;
 }
 
 // n / d for 32-bit n by multiply-high and shifts (Granlund-Montgomery).
@@ -244,6 +280,7 @@ __device__ __forceinline__ uint32_t fast_div(uint32_t n, const FastDiv& d) {
 #ifndef NVFP4_QMINB
 #define NVFP4_QMINB 1
 #endif
+
 
 // Dynamic (per-call) global scale inside the sweep launch: every CTA folds the
 // max |x| of its grid-stride share into one partial, all CTAs meet at a grid
@@ -459,7 +496,8 @@ __global__ void __launch_bounds__(256, quantize_min_blocks<METHOD, DT>()) quanti
             const int I0 = e4m3_floor_code(sbase);
             if (FIX) {
                 const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
-                bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK>(y2, w2, m, tb, best);
+                bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK>(y2, w2, m, tb, best,
+                                                                         OBJ == 0 || weights_nonneg(w2));
             } else {
                 int lo_off = p.win_lo;
                 if ((p.tight & 2) && I0 >= 16 && I0 <= 120) {
