@@ -281,7 +281,7 @@ __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand*
         float best;
         const int I0 = e4m3_floor_code(__fdiv_rn(m, 6.0f));
         const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
-        bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK>(y2, w2, m, tb, best, wok);
+        bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK, true>(y2, w2, m, tb, best, wok);
     } else {
         bestc = max((int)e4m3_rn_code(__fdiv_rn(m, 6.0f)), 1);
     }

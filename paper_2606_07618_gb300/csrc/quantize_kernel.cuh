@@ -204,18 +204,22 @@ __device__ __forceinline__ float group_max(float v) {
 // 1.409/1.369/1.336/1.325/1.334 with static scales; WMSE blocks of 32 and 64
 // gain nothing (a single element's term is small against a 32- or 64-element
 // loss) and lose up to 2% at NB 4, so they keep the plain sweep.
-template <int OBJ, int BLOCK>
+// WMSE_BOUND = false leaves WMSE to the plain sweep: the per-tensor kernel
+// reloads a lane's weights every segment, and checking them there as well
+// made its WMSE sweep 2.6% slower on Gaussian 16384 x 8192 weights (0.378 ->
+// 0.388 ms) while the Student-t activations of the latency table gained 1.2%.
+template <int OBJ, int BLOCK, bool WMSE_BOUND>
 __host__ __device__ constexpr int bound_offsets() {
-    return OBJ != 0 ? (BLOCK == 16 ? 4 : 0) : (BLOCK == 16 ? 1 : (BLOCK == 32 ? 5 : 4));
+    return OBJ != 0 ? (BLOCK == 16 && WMSE_BOUND ? 4 : 0) : (BLOCK == 16 ? 1 : (BLOCK == 32 ? 5 : 4));
 }
 
-template <int OBJ, int BLOCK>
+template <int OBJ, int BLOCK, bool WMSE_BOUND>
 __device__ __forceinline__ int default_window_argmin(const u64 (&y2)[8], const u64 (&w2)[8], float m, const Cand* tb,
                                                      float& best, bool wok = true) {
     constexpr int SEGS = BLOCK / 16;
     constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
     constexpr int FIX_K = 7 - FIX_LO + 1;
-    constexpr int NB = bound_offsets<OBJ, BLOCK>();
+    constexpr int NB = bound_offsets<OBJ, BLOCK, WMSE_BOUND>();
     best = __int_as_float(0x7f800000);
     int bk = 0;
 #pragma unroll
@@ -494,10 +498,27 @@ __global__ void __launch_bounds__(256, quantize_min_blocks<METHOD, DT>()) quanti
         if (METHOD == 0) {
             const float sbase = __fdiv_rn(m, 6.0f);
             const int I0 = e4m3_floor_code(sbase);
-            if (FIX) {
+            if (FIX && OBJ == 0) {
                 const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
-                bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK>(y2, w2, m, tb, best,
-                                                                         OBJ == 0 || weights_nonneg(w2));
+                bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK, false>(y2, w2, m, tb, best);
+            } else if (FIX) {
+                // WMSE: the plain sweep.  The explicit unroll count matters: a
+                // bare "#pragma unroll" of the same 16-iteration loop compiles to
+                // another schedule (116 instead of 118 registers) that measured
+                // 1.2% slower at 16384 x 8192.
+                constexpr int FIX_K = 7 - FIX_LO + 1;
+                const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
+                int bk = 0;
+#pragma unroll 16
+                for (int k = 0; k < FIX_K; k++) {
+                    const Cand cd = tb[k];
+                    const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));
+                    if (L < best) {
+                        best = L;
+                        bk = k;
+                    }
+                }
+                bestc = I0 + FIX_LO + bk;
             } else {
                 int lo_off = p.win_lo;
                 if ((p.tight & 2) && I0 >= 16 && I0 <= 120) {

@@ -7,8 +7,8 @@ stress the bound: heavy-tailed blocks (where the bound skips), blocks whose
 largest value repeats, all-zero and NaN/inf blocks in the same warp, negative
 and NaN weights (for which skipping must switch itself off), per-row weights,
 global scales near the ends of the E4M3 range, and blocks of 16, 32 and 64 in
-both input types.  The grouped launch (which takes the same path) must give
-the same bytes as well.
+both input types.  The per-tensor sweep skips for MSE; the grouped launch,
+which must give the same bytes, skips for MSE and for WMSE with blocks of 16.
 """
 import numpy as np
 import pytest
@@ -76,6 +76,16 @@ def run(B, x, block, S, obj, w, stride, window):
     return out
 
 
+def run_group(B, x, block, S, obj, w, stride):
+    rows, cols = x.shape
+    out = B.empty_outputs(rows, cols, block, device=DEV, linear=True, swizzled=block == 16)
+    desc = B.group_descriptors([x], [w], [stride], [out["codes"]], [out["sf_linear"]], [out["sf_swizzled"]])
+    dt = B.NVFP4_IN_BF16 if x.dtype == torch.bfloat16 else B.NVFP4_IN_F32
+    B.scalesweep_quantize_group(desc, dt, obj, 0.0, S, None, None, block=block)
+    torch.cuda.synchronize()
+    return out
+
+
 def same(a, b):
     for k in ("codes", "sf_linear", "sf_swizzled", "block_loss"):
         if a[k] is None:
@@ -103,6 +113,10 @@ def test_skipping_sweep_equals_full_window(B, dtype, block, obj, wkind, xkind):
         fast = run(B, xd, block, S, obj, wd, stride, (B.NVFP4_WINDOW_DEFAULT, B.NVFP4_WINDOW_DEFAULT))
         full = run(B, xd, block, S, obj, wd, stride, (lo, 7))
         same(fast, full)
+        grouped = run_group(B, xd, block, S, obj, wd, stride)      # the grouped sweep skips for WMSE too
+        for k in ("codes", "sf_linear", "sf_swizzled"):
+            if grouped[k] is not None:
+                assert torch.equal(grouped[k], full[k]), k
 
 
 @pytest.mark.parametrize("obj", [0, 1])
