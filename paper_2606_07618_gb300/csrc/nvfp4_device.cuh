@@ -70,24 +70,6 @@ __device__ __forceinline__ u64 cand_err2(u64 y2, u64 r2, uint16_t nv) {
     return e2;
 }
 
-// The same candidate step on one element: e = fl(y - q*v) with q =
-// RNE_E2M1(fl(y*r)), bit for bit the value cand_err2 gives that element.
-__device__ __forceinline__ float cand_err1(float y, float r, uint16_t nv) {
-    float e;
-    asm("{\n\t"
-        ".reg .b32 t, h2;\n\t"
-        ".reg .b16 ql, qh;\n\t"
-        ".reg .b8 q;\n\t"
-        "mul.rn.f32 t, %1, %2;\n\t"
-        "cvt.rn.satfinite.e2m1x2.f32 q, t, t;\n\t"
-        "cvt.rn.f16x2.e2m1x2 h2, q;\n\t"
-        "mov.b32 {ql, qh}, h2;\n\t"
-        "fma.rn.f32.f16 %0, ql, %3, %1;\n\t"
-        "}"
-        : "=f"(e) : "f"(y), "f"(r), "h"(nv));
-    return e;
-}
-
 // E4M3 code -> f16 bit pattern of its value (exact), via the native decode.
 __device__ __forceinline__ uint16_t e4m3_to_f16bits(uint32_t code) {
     uint32_t h2;

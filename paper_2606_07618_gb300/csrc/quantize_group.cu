@@ -240,9 +240,9 @@ __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand*
     constexpr int SEGS = BLOCK / 16;
     constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
     u64 y2[8];
-    float m = 0.0f;
+    float m = 0.0f, ma = 0.0f, mb = 0.0f;               // ma, mb: largest |y| of each half (offset bound)
     if (valid) {
-        m = raw_to_y<DT>(cur, E2, y2);
+        m = METHOD == 0 ? raw_to_y_halves<DT>(cur, E2, y2, ma, mb) : raw_to_y<DT>(cur, E2, y2);
     } else {
 #pragma unroll
         for (int j = 0; j < 8; j++) y2[j] = 0ull;
@@ -281,7 +281,7 @@ __device__ __forceinline__ void sweep_segments(const GroupTensor& d, const Cand*
         float best;
         const int I0 = e4m3_floor_code(__fdiv_rn(m, 6.0f));
         const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
-        bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK, true>(y2, w2, m, tb, best, wok);
+        bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK, true>(y2, w2, ma, mb, tb, best, wok);
     } else {
         bestc = max((int)e4m3_rn_code(__fdiv_rn(m, 6.0f)), 1);
     }

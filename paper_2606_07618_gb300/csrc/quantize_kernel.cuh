@@ -146,6 +146,38 @@ __device__ __forceinline__ float raw_to_y(const Raw& r, u64 E2, u64 (&y2)[8]) {
     return max3f(max3f(p0, p1, p2), max3f(p3, p4, av[15]), 0.0f);
 }
 
+// raw_to_y that also returns the largest |y| of each half of the segment
+// (elements 0-7 in ma, 8-15 in mb); m = max(ma, mb) is raw_to_y's value.
+template <int DT>
+__device__ __forceinline__ float raw_to_y_halves(const Raw& r, u64 E2, u64 (&y2)[8], float& ma, float& mb) {
+    uint32_t u[16];
+    if (DT == 0) {
+        const uint32_t p[8] = {r.a.x, r.a.y, r.a.z, r.a.w, r.b.x, r.b.y, r.b.z, r.b.w};
+#pragma unroll
+        for (int j = 0; j < 8; j++) {
+            u[2 * j] = p[j] << 16;
+            u[2 * j + 1] = p[j] & 0xFFFF0000u;
+        }
+    } else {
+        const uint32_t p[16] = {r.a.x, r.a.y, r.a.z, r.a.w, r.b.x, r.b.y, r.b.z, r.b.w,
+                                r.c.x, r.c.y, r.c.z, r.c.w, r.d.x, r.d.y, r.d.z, r.d.w};
+#pragma unroll
+        for (int j = 0; j < 16; j++) u[j] = p[j];
+    }
+    float av[16];
+#pragma unroll
+    for (int j = 0; j < 8; j++) {
+        y2[j] = mul2(pack2(__uint_as_float(u[2 * j]), __uint_as_float(u[2 * j + 1])), E2);
+        float a, b;
+        unpack2(y2[j], a, b);
+        av[2 * j] = fabsf(a);
+        av[2 * j + 1] = fabsf(b);
+    }
+    ma = max3f(max3f(av[0], av[1], av[2]), max3f(av[3], av[4], av[5]), max2f(av[6], av[7]));
+    mb = max3f(max3f(av[8], av[9], av[10]), max3f(av[11], av[12], av[13]), max2f(av[14], av[15]));
+    return max3f(ma, mb, 0.0f);
+}
+
 // Loss of one candidate on this thread's 16 elements.
 template <int OBJ>
 __device__ __forceinline__ float seg_loss(const u64 (&y2)[8], const u64 (&w2)[8], float r, uint16_t nv) {
@@ -184,38 +216,56 @@ __device__ __forceinline__ float group_max(float v) {
 // whose loss is minimal and sets `best` to that loss.
 //
 // The lowest NB offsets are visited last, in descending order, and a warp
-// skips one when, for every lane, the block's largest element alone already
-// costs more than the lane's best loss so far.  That single term -- fl(e_m^2)
-// for MSE, fl(fl(w_m e_m) e_m) for WMSE, with e_m = cand_err1(m, ...) and w_m
-// the weight of an element whose |y| is m -- is the term the candidate's loss
-// accumulates for that element, every other term is non-negative (squares;
-// WMSE: only while the lane's weights are non-negative, `wok`, else no skip),
-// and rounding is monotone, so the loss is at least the term: a skipped
-// candidate has a loss above the final best and can neither win nor tie.  The
-// losses that are computed are the same values in the same order, with ties
-// going to the lowest code (<= for the codes below every code already
-// visited), so the result is the full sweep's, bit for bit.  On the low
-// offsets the block's largest element saturates (6 v_c < m), which makes the
-// bound tight: on the synthetic Qwen2.5-72B-shaped weights a warp skips offset
-// 0 of the 11 MSE candidates (I0-3) in 96% of its visits, ~5 of the 16 MSE
-// candidates of blocks of 32/64, and ~2.4 of the 16 WMSE candidates of blocks
-// of 16.  NB per objective and block as measured on those weights (grouped
-// call, ms; every NB gave the same output bytes): WMSE block 16, NB 0/2/3/4/5:
-// 1.409/1.369/1.336/1.325/1.334 with static scales; WMSE blocks of 32 and 64
-// gain nothing (a single element's term is small against a 32- or 64-element
-// loss) and lose up to 2% at NB 4, so they keep the plain sweep.
-// WMSE_BOUND = false leaves WMSE to the plain sweep: the per-tensor kernel
-// reloads a lane's weights every segment, and checking them there as well
-// made its WMSE sweep 2.6% slower on Gaussian 16384 x 8192 weights (0.378 ->
-// 0.388 ms) while the Student-t activations of the latency table gained 1.2%.
+// skips one when, for every lane, a lower bound on the block's loss for that
+// candidate already exceeds the lane's best loss so far.  The bound is the sum
+// of two terms per lane of the block, those of the largest |y| of each half of
+// the lane's segment (ma, mb: distinct elements), computed with the loop's own
+// arithmetic: cand_err2 gives their errors e bit for bit and the terms are
+// fl(e e) (MSE) or fl(fl(w e) e) (WMSE, w the weight of an element of that
+// half whose |y| is its maximum).  The loss accumulates every element's
+// product exactly once into a rounded running sum, so with non-negative terms
+// (squares; WMSE: only while the lane's weights are non-negative, `wok`, else
+// no skip) and monotone rounding it is at least the two products' sum with at
+// most four roundings (two in a lane, two in the block's shuffle sum), while
+// the bound is computed with at most six upward roundings and then multiplied
+// by 1 - 2^-20, which covers both: a skipped candidate's loss is above the
+// final best, so it can neither win nor tie.  The losses that are computed are
+// the same values in the same order, with ties going to the lowest code (<=
+// for the codes below every code already visited), so the result is the full
+// sweep's, bit for bit.  On the low offsets the largest elements saturate
+// (6 v_c < m), which makes the bound tight.  A CPU simulation on the synthetic
+// Qwen2.5-72B-shaped weights (warps of 32 consecutive blocks) gives the skips
+// per warp: WMSE 3.4 of 16 candidates with blocks of 16 (NB 4; 2.2 with the
+// largest element alone), 3.4 / 3.3 with blocks of 32 / 64 (NB 4); MSE 1.2 of
+// 11 with blocks of 16 (NB 2), 5.9 / 5.5 of 16 with blocks of 32 / 64 (NB 6).
+// NB measured on the grouped call over the full workloads (ms, in-launch
+// scales; every setting gave the same output bytes), WMSE16/WMSE32,64/MSE16/
+// MSE32,64 = 4/0/1/5, 5/4/2/6, 6/6/3/7: Qwen shapes WMSE block 16
+// 1.369/1.369/1.386, block 32 1.502/1.390/1.390, block 64 1.558/1.433/1.454;
+// MSE block 16 0.869/0.863/0.886, block 32 0.991/0.954/0.973, block 64
+// 1.034/0.997/1.022; Llama-3-8B layer 0.620/0.623/0.632 (no bound: 1.511 Qwen
+// WMSE block 16, 0.684 Llama, 0.892 Qwen MSE block 16).
+#ifndef NVFP4_NB_WMSE16
+#define NVFP4_NB_WMSE16 4
+#endif
+#ifndef NVFP4_NB_WMSE3264
+#define NVFP4_NB_WMSE3264 4
+#endif
+#ifndef NVFP4_NB_MSE16
+#define NVFP4_NB_MSE16 2
+#endif
+#ifndef NVFP4_NB_MSE3264
+#define NVFP4_NB_MSE3264 6
+#endif
 template <int OBJ, int BLOCK, bool WMSE_BOUND>
 __host__ __device__ constexpr int bound_offsets() {
-    return OBJ != 0 ? (BLOCK == 16 && WMSE_BOUND ? 4 : 0) : (BLOCK == 16 ? 1 : (BLOCK == 32 ? 5 : 4));
+    return OBJ != 0 ? (WMSE_BOUND ? (BLOCK == 16 ? NVFP4_NB_WMSE16 : NVFP4_NB_WMSE3264) : 0)
+                    : (BLOCK == 16 ? NVFP4_NB_MSE16 : NVFP4_NB_MSE3264);
 }
 
 template <int OBJ, int BLOCK, bool WMSE_BOUND>
-__device__ __forceinline__ int default_window_argmin(const u64 (&y2)[8], const u64 (&w2)[8], float m, const Cand* tb,
-                                                     float& best, bool wok = true) {
+__device__ __forceinline__ int default_window_argmin(const u64 (&y2)[8], const u64 (&w2)[8], float ma, float mb,
+                                                     const Cand* tb, float& best, bool wok = true) {
     constexpr int SEGS = BLOCK / 16;
     constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
     constexpr int FIX_K = 7 - FIX_LO + 1;
@@ -232,28 +282,33 @@ __device__ __forceinline__ int default_window_argmin(const u64 (&y2)[8], const u
         }
     }
     if (NB == 0) return bk;
-    float wm = 1.0f;
+    const u64 m2 = pack2(ma, mb);
+    u64 wab = 0ull;
     if (OBJ == 1) {
-        // weight of an element of this lane whose |y| is the block max (0 if
-        // none), then the largest over the block's lanes: every element at the
-        // max has the same error, so any of their weights gives a valid term
-        wm = 0.0f;
+        // the weight of an element of each half whose |y| is that half's max
+        float wa = 0.0f, wb = 0.0f;
 #pragma unroll
         for (int j = 0; j < 8; j++) {
-            float a, b, wa, wb;
+            float a, b, w0, w1;
             unpack2(y2[j], a, b);
-            unpack2(w2[j], wa, wb);
-            wm = fabsf(a) == m ? wa : wm;
-            wm = fabsf(b) == m ? wb : wm;
+            unpack2(w2[j], w0, w1);
+            float& wh = j < 4 ? wa : wb;
+            const float mh = j < 4 ? ma : mb;
+            wh = fabsf(a) == mh ? w0 : wh;
+            wh = fabsf(b) == mh ? w1 : wh;
         }
-        wm = group_max<SEGS>(wok ? wm : __int_as_float(0x7fc00000));   // negative or NaN weights: no skip
+        if (!wok) wa = __int_as_float(0x7fc00000);     // negative or NaN weights: no skip
+        wab = pack2(wa, wb);
     }
 #pragma unroll
     for (int k = NB - 1; k >= 0; k--) {
         const Cand cd = tb[k];
-        const float e = cand_err1(m, cd.r, (uint16_t)cd.nv);
-        const float term = OBJ == 1 ? __fmul_rn(__fmul_rn(wm, e), e) : __fmul_rn(e, e);
-        if (__all_sync(0xffffffffu, term > best)) continue;                  // warp-uniform
+        const u64 e2 = cand_err2(m2, pack2(cd.r, cd.r), (uint16_t)cd.nv);
+        const u64 t2 = OBJ == 1 ? mul2(mul2(wab, e2), e2) : mul2(e2, e2);
+        float ta, tb2;
+        unpack2(t2, ta, tb2);
+        const float bound = __fmul_rn(group_sum<SEGS>(__fadd_rn(ta, tb2)), 0.99999904632568359375f);
+        if (__all_sync(0xffffffffu, bound > best)) continue;                  // warp-uniform
         const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));
         if (L <= best) {
             best = L;
@@ -450,9 +505,9 @@ __global__ void __launch_bounds__(256, quantize_min_blocks<METHOD, DT>()) quanti
         if (g + stride < p.nseg) load_raw<DT>(p.x, g + stride, nxt);
 
         u64 y2[8];
-        float m = 0.0f;
+        float m = 0.0f, ma = 0.0f, mb = 0.0f;         // ma, mb: largest |y| of each half (offset bound)
         if (valid) {
-            m = raw_to_y<DT>(cur, E2, y2);
+            m = METHOD == 0 ? raw_to_y_halves<DT>(cur, E2, y2, ma, mb) : raw_to_y<DT>(cur, E2, y2);
         } else {
 #pragma unroll
             for (int j = 0; j < 8; j++) y2[j] = 0ull;
@@ -500,7 +555,7 @@ __global__ void __launch_bounds__(256, quantize_min_blocks<METHOD, DT>()) quanti
             const int I0 = e4m3_floor_code(sbase);
             if (FIX && OBJ == 0) {
                 const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
-                bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK, false>(y2, w2, m, tb, best);
+                bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK, false>(y2, w2, ma, mb, tb, best);
             } else if (FIX) {
                 // WMSE: the plain sweep.  The explicit unroll count matters: a
                 // bare "#pragma unroll" of the same 16-iteration loop compiles to
