@@ -41,9 +41,9 @@
 // CTAs on the registers they leave free: the largest tensor is reduced, then
 // swept while the other tensors are reduced beside it, then the others are
 // swept.  Only the first reduction is exposed.  On the two Qwen2.5-72B-shaped
-// matrices (WMSE) 1.506-1.512 ms per call against 1.568-1.573 ms two-phase and
-// 1.406-1.411 ms with static scales; on the Llama-3-8B layer 0.681 against
-// 0.735 (static 0.643).
+// matrices (WMSE, full-window sweep) 1.506-1.512 ms per call against
+// 1.568-1.573 ms two-phase and 1.406-1.411 ms with static scales; on the
+// Llama-3-8B layer 0.681 against 0.735 (static 0.643).
 #include <atomic>
 
 #include "group_kernels.h"
