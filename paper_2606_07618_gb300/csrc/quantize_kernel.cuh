@@ -245,31 +245,27 @@ __device__ __forceinline__ float group_max(float v) {
 // MSE block 16 0.869/0.863/0.886, block 32 0.991/0.954/0.973, block 64
 // 1.034/0.997/1.022; Llama-3-8B layer 0.620/0.623/0.632 (no bound: 1.511 Qwen
 // WMSE block 16, 0.684 Llama, 0.892 Qwen MSE block 16).
-#ifndef NVFP4_NB_WMSE16
-#define NVFP4_NB_WMSE16 4
-#endif
-#ifndef NVFP4_NB_WMSE3264
-#define NVFP4_NB_WMSE3264 4
-#endif
-#ifndef NVFP4_NB_MSE16
-#define NVFP4_NB_MSE16 2
-#endif
-#ifndef NVFP4_NB_MSE3264
-#define NVFP4_NB_MSE3264 6
-#endif
-template <int OBJ, int BLOCK, bool WMSE_BOUND>
+// GROUPED: the grouped kernel (else the per-tensor one), whose best MSE
+// block-16 setting differs (per-tensor sweeps, ms, NB 1 against 2: Gaussian
+// 16384 x 8192 0.2125/0.218, Student-t 32768 x 8192 0.4154/0.4219, Laplace
+// 8192 x 8192 0.1085/0.1104; per-tensor WMSE with NB 4 against the plain
+// sweep: 0.3585/0.3831, 0.704/0.757, 0.1815/0.1947).  Per-tensor blocks of
+// 32/64 on the same three tensors, MSE NB 6/5/4/0: 0.266/0.274/0.278/0.303 and
+// 0.287/0.279/0.289/0.318 (Gaussian), 0.522/0.542/0.550/0.592 and
+// 0.547/0.550/0.572/0.630 (Student-t); WMSE NB 4 against 0: 0.381/0.391 and
+// 0.387/0.389 (Gaussian), 0.753/0.776 and 0.764/0.764 (Student-t).
+template <int OBJ, int BLOCK, bool GROUPED>
 __host__ __device__ constexpr int bound_offsets() {
-    return OBJ != 0 ? (WMSE_BOUND ? (BLOCK == 16 ? NVFP4_NB_WMSE16 : NVFP4_NB_WMSE3264) : 0)
-                    : (BLOCK == 16 ? NVFP4_NB_MSE16 : NVFP4_NB_MSE3264);
+    return OBJ != 0 ? 4 : (BLOCK == 16 ? (GROUPED ? 2 : 1) : 6);
 }
 
-template <int OBJ, int BLOCK, bool WMSE_BOUND>
+template <int OBJ, int BLOCK, bool GROUPED>
 __device__ __forceinline__ int default_window_argmin(const u64 (&y2)[8], const u64 (&w2)[8], float ma, float mb,
                                                      const Cand* tb, float& best, bool wok = true) {
     constexpr int SEGS = BLOCK / 16;
     constexpr int FIX_LO = (OBJ == 0 && BLOCK == 16) ? -3 : -8;
     constexpr int FIX_K = 7 - FIX_LO + 1;
-    constexpr int NB = bound_offsets<OBJ, BLOCK, WMSE_BOUND>();
+    constexpr int NB = bound_offsets<OBJ, BLOCK, GROUPED>();
     best = __int_as_float(0x7f800000);
     int bk = 0;
 #pragma unroll
@@ -553,27 +549,12 @@ __global__ void __launch_bounds__(256, quantize_min_blocks<METHOD, DT>()) quanti
         if (METHOD == 0) {
             const float sbase = __fdiv_rn(m, 6.0f);
             const int I0 = e4m3_floor_code(sbase);
-            if (FIX && OBJ == 0) {
+            if (FIX) {
+                // the lane's weights are reloaded every segment, so their signs
+                // are checked every segment too
                 const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
-                bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK, false>(y2, w2, ma, mb, tb, best);
-            } else if (FIX) {
-                // WMSE: the plain sweep.  The explicit unroll count matters: a
-                // bare "#pragma unroll" of the same 16-iteration loop compiles to
-                // another schedule (116 instead of 118 registers) that measured
-                // 1.2% slower at 16384 x 8192.
-                constexpr int FIX_K = 7 - FIX_LO + 1;
-                const Cand* tb = tab + (I0 + FIX_LO + kTabOff);
-                int bk = 0;
-#pragma unroll 16
-                for (int k = 0; k < FIX_K; k++) {
-                    const Cand cd = tb[k];
-                    const float L = group_sum<SEGS>(seg_loss<OBJ>(y2, w2, cd.r, (uint16_t)cd.nv));
-                    if (L < best) {
-                        best = L;
-                        bk = k;
-                    }
-                }
-                bestc = I0 + FIX_LO + bk;
+                bestc = I0 + FIX_LO + default_window_argmin<OBJ, BLOCK, false>(y2, w2, ma, mb, tb, best,
+                                                                               OBJ == 0 || weights_nonneg(w2));
             } else {
                 int lo_off = p.win_lo;
                 if ((p.tight & 2) && I0 >= 16 && I0 <= 120) {
