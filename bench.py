@@ -326,7 +326,8 @@ def run_gpu(args, rank, world):
                 f"({len(xs)} tensors, one launch per step)",
                 "peak_note": f"{nsm} SMs x 128 FP32 lanes x median SM clock {sm_mhz} MHz "
                              f"(of measured clock; the work is {alu_ops_per_elem(wl)} FP32 ops per element: "
-                             f"{candidates(wl)} candidates x 4)",
+                             f"{candidates(wl)} candidates x 4, counted for every window candidate, including "
+                             f"those the sweep's exact offset bound rules out without evaluating them)",
                 "hbm": {"achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": hfrac, "peak_kind": peak_kind,
                         "bytes": round(hbm_bytes(wl, xs)), "bytes_per_elem": round(hbm_bytes(wl, xs) / total, 4)},
                 "launch_ms": round(kern_ms, 4),
