@@ -211,10 +211,10 @@ __device__ __forceinline__ bool grid_barrier(const GroupParams& p) {
 // scheduled once every CTA of that sweep is resident, reads only its own
 // tensors, and ends with griddepcontrol.wait, so it completes (and the next
 // sweep, which waits for it, starts) only after that sweep has completed.
-template <int DT>
-__global__ void __launch_bounds__(kReduceThreads, 2048 / kReduceThreads)
+template <int DT, int THREADS = kReduceThreads, int INFLIGHT = kReduceInFlight>
+__global__ void __launch_bounds__(THREADS, 2048 / THREADS)
     group_reduce_kernel(const __grid_constant__ GroupParams p, unsigned* ticket) {
-    reduce_all<DT, kReduceInFlight, kReduceThreads>(p);
+    reduce_all<DT, INFLIGHT, THREADS>(p);
     __syncthreads();                                 // every warp's atomics are fenced
     if (threadIdx.x == 0 && atom_add_acq_rel(ticket, 1u) == gridDim.x - 1) {
         for (int a = 0; a < p.count; a++)            // the last CTA sees every CTA's maxima
@@ -528,7 +528,9 @@ cudaError_t launch_group_pipelined(const GroupParams& p, int sms, cudaStream_t s
     unsigned* ticket = p.arrived;
     cudaError_t e = cudaMemsetAsync(p.amax_bits, 0, kGroupWorkspace, s);
     if (e != cudaSuccess) return e;
-    group_reduce_kernel<DT><<<(unsigned)sms * (2048 / kReduceThreads), kReduceThreads, 0, s>>>(a, ticket);
+    // the first reduction has the GPU to itself: 512-thread CTAs, 4 per SM, 8
+    // loads in flight per lane (0.2-0.4% faster steps than the 128-thread form)
+    group_reduce_kernel<DT, 512, 8><<<(unsigned)sms * 4, 512, 0, s>>>(a, ticket);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     int occ = 1;
     const bool big_rest = b.total_seg > a.total_seg / 2;
@@ -553,6 +555,7 @@ cudaError_t launch_group_pipelined(const GroupParams& p, int sms, cudaStream_t s
     const int free_per_sched = 16384 - sweep_warps_per_sched * warp_regs;
     int per_sm = free_per_sched / (32 * 32) / (kReduceThreads / 32 / 4);
     per_sm = per_sm < 1 ? 1 : (per_sm > 2048 / kReduceThreads ? 2048 / kReduceThreads : per_sm);
+
     e = launch_dependent(group_reduce_kernel<DT>, (int64_t)sms * per_sm, kReduceThreads, s, b, ticket + 1);
     if (e != cudaSuccess) return e;
     const int64_t grid_b = sweep_grid<DT, METHOD, OBJ, BLOCK, 2>(b, sms, nullptr);
