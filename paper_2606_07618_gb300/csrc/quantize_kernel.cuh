@@ -149,7 +149,7 @@ __device__ __forceinline__ float raw_to_y(const Raw& r, u64 E2, u64 (&y2)[8]) {
 // raw_to_y that also returns the largest |y| of each half of the segment
 // (elements 0-7 in ma, 8-15 in mb); m = max(ma, mb) is raw_to_y's value.  Its
 // max tree takes one more instruction than raw_to_y's, which the methods that
-// have no use for the halves (AbsMax, 4/6, custom windows) therefore keep.
+// have no use for the halves (AbsMax, 4/6) therefore keep.
 template <int DT>
 __device__ __forceinline__ float raw_to_y_halves(const Raw& r, u64 E2, u64 (&y2)[8], float& ma, float& mb) {
     uint32_t u[16];
