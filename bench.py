@@ -513,7 +513,9 @@ def run_e2e(wl, xs, ws, dev, stream, world, args):
         torch.cuda.synchronize()
         return a.elapsed_time(b) / reps
 
-    e_reps = max(3, min(10, args.steps))
+    # 30 steps per trial: the pipeline's fill and drain (one step's compute and
+    # download) then cost ~1/30 of a step each, not 1/10
+    e_reps = max(3, min(30, args.steps))
     total = sum(x.numel() for x in xs)
     h2d = sum(x.numel() * x.element_size() for x in xs)
     d2h = sum(h.numel() * h.element_size() for d in hout for h in d.values())
